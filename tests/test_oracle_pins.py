@@ -1,0 +1,517 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Nothing here re-types the oracle's formulas: each check compares the
+oracle's output with an independent statement -- a theorem or lemma of the
+paper evaluated in exact rational arithmetic, a brute-force search over the
+grid, a hand-worked fixture, or an independent library routine (numpy's
+float16 conversion, numpy's float64 matmul).
+"""
+import itertools
+import os
+from fractions import Fraction as F
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2607_08779_gb300 import inputs
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+QS = (2, 3, 4)
+GRID_CODE = {"U": oracle.GRID_UNSIGNED_SYM, "S": oracle.GRID_SIGNED_SYM,
+             "A": oracle.GRID_ASYM}
+
+
+def alphabet(q):
+    """A_q = {-2^(q-1), ..., 2^(q-1)-1} (Sec. 1, Notation)."""
+    return range(-(1 << (q - 1)), 1 << (q - 1))
+
+
+def nearest_index(w: F, base: F, step: F, idx):
+    """Brute force: the a in idx minimising |w - (base + step*a)|; an exact
+    tie between two neighbours goes to the even a."""
+    best = None
+    for a in idx:
+        d = abs(w - (base + step * a))
+        if best is None or d < best[0] or (d == best[0] and a % 2 == 0):
+            best = (d, a)
+    return best[1]
+
+
+def is_midpoint(x: F) -> bool:
+    return (x - F(1, 2)).denominator == 1
+
+
+def dominant_outlier(w):
+    """(index, value) of the largest-magnitude coordinate following the sign
+    rule's reading: positive if max w > -min w, else negative."""
+    mx, mn = float(np.max(w)), float(np.min(w))
+    i = int(np.argmax(w)) if mx > -mn else int(np.argmin(w))
+    return i, float(w[i])
+
+
+def random_groups(n, g, seed, outliers=True):
+    w = inputs.student_t_weights(n, g, seed, outliers=False)
+    if outliers:
+        # plant a few large coordinates, of random sign, as the outlier channels do
+        rng = np.random.default_rng(seed)
+        rows = rng.random(n) < 0.5
+        cols = rng.integers(0, g, n)
+        w[rows, cols[rows]] *= 20.0
+    return w
+
+
+def lattice_groups(d, den):
+    vals = [F(i, den) for i in range(-den, den + 1)]
+    for combo in itertools.product(vals, repeat=d):
+        if any(v != 0 for v in combo):
+            yield np.array([float(v) for v in combo], np.float32)
+
+
+# --------------------------------------------------------------------------
+# IEEE binary16 (the stored scale format of the Q-formats, Appendix)
+# --------------------------------------------------------------------------
+
+def test_f32_to_f16_matches_numpy():
+    rng = np.random.default_rng(1)
+    vals = list(rng.standard_normal(4000).astype(np.float32))
+    vals += list((rng.standard_normal(4000) * 2.0 ** rng.integers(-30, 20, 4000))
+                 .astype(np.float32))
+    edges = [0.0, -0.0, 65504.0, 65519.0, 65519.99, 65520.0, -65520.0, 1e9,
+             2.0 ** -24, 2.0 ** -25, 3 * 2.0 ** -26, 2.0 ** -14, 2.0 ** -15,
+             (1 + 2.0 ** -11) * 2.0 ** -14, 1 + 2.0 ** -11, 1 + 3 * 2.0 ** -11,
+             np.inf, -np.inf, 1e-40]
+    vals += [np.float32(e) for e in edges]
+    for x in vals:
+        with np.errstate(over="ignore"):
+            want = int(np.array([x], np.float32).astype(np.float16).view(np.uint16)[0])
+        assert oracle.f32_to_f16(x) == want, x
+
+
+def test_f16_to_f32_exhaustive():
+    bits = np.arange(1 << 16, dtype=np.uint32).astype(np.uint16)
+    ref = bits.view(np.float16).astype(np.float32)
+    got = np.array([oracle.f16_to_f32(int(b)) for b in bits], np.float32)
+    nan = np.isnan(ref)
+    assert np.array_equal(np.isnan(got), nan)
+    assert np.array_equal(got[~nan].view(np.uint32), ref[~nan].view(np.uint32))
+
+
+# --------------------------------------------------------------------------
+# Hand-worked fixtures and the paper's printed block sizes
+# --------------------------------------------------------------------------
+
+def _golden_records():
+    for line in open(os.path.join(GOLDEN, "hand_groups.txt")):
+        line = line.strip()
+        if not line or line.startswith("#"):
+            continue
+        f = [x.strip() for x in line.split("|")]
+        yield {
+            "q": int(f[0]), "grid": GRID_CODE[f[1]],
+            "w": np.array([float(v) for v in f[2].split()], np.float32),
+            "c": [int(v) for v in f[3].split()],
+            "u": [int(v) for v in f[4].split()],
+            "s32": float(f[5]), "s16": int(f[6], 16),
+            "m16": None if f[7] == "-" else int(f[7], 16),
+            "packed": bytes.fromhex(f[8]),
+        }
+
+
+@pytest.mark.parametrize("rec", list(_golden_records()), ids=lambda r: f"q{r['q']}g{r['grid']}")
+def test_hand_worked_groups(rec):
+    r = oracle.quantize_group(rec["w"], rec["q"], rec["grid"])
+    assert list(r["c"]) == rec["c"]
+    assert list(r["u"]) == rec["u"]
+    assert r["s32"] == rec["s32"]
+    assert r["s16"] == rec["s16"]
+    if rec["m16"] is not None:
+        assert r["m16"] == rec["m16"]
+    assert bytes(oracle.pack_group(r["u"], rec["q"])) == rec["packed"]
+
+
+def test_paper_block_sizes():
+    w = inputs.student_t_weights(1, 32, 7)
+    for line in open(os.path.join(GOLDEN, "paper_block_sizes.txt")):
+        if line.startswith("#") or not line.strip():
+            continue
+        q, kind, nbytes = [x.strip() for x in line.split("|")]
+        q, nbytes = int(q), int(nbytes)
+        grid = oracle.GRID_ASYM if kind == "asym" else oracle.GRID_SIGNED_SYM
+        codes, scales, mins, _, _ = oracle.quantize(w, q, 32, grid)
+        total = codes.nbytes + scales.nbytes + (mins.nbytes if mins is not None else 0)
+        assert total == nbytes
+
+
+# --------------------------------------------------------------------------
+# eq:quantizer: rounding to nearest and clipping, by brute force
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("q", QS)
+@pytest.mark.parametrize("d,den", [(2, 16), (3, 8)])
+def test_symmetric_codes_are_nearest_grid_points(q, d, den):
+    """Exhaustive dyadic lattice, both scale signs, exact ties included."""
+    A = alphabet(q)
+    for w in lattice_groups(d, den):
+        for gamma in (1, -1):
+            r = oracle.quantize_group_gamma(w, q, gamma)
+            s = F(r["s32"])
+            for j in range(d):
+                assert r["c"][j] == nearest_index(F(float(w[j])), F(0), s, A)
+                assert r["u"][j] == r["c"][j] + (1 << (q - 1))
+
+
+@pytest.mark.parametrize("q", QS)
+@pytest.mark.parametrize("g", [32, 128])
+def test_symmetric_codes_random_groups(q, g):
+    A = alphabet(q)
+    W = random_groups(40, g, 11 * q + g)
+    for w in W:
+        for grid in (oracle.GRID_UNSIGNED_SYM, oracle.GRID_SIGNED_SYM):
+            r = oracle.quantize_group(w, q, grid)
+            s = F(r["s32"])
+            for j in range(g):
+                assert r["c"][j] == nearest_index(F(float(w[j])), F(0), s, A)
+
+
+# --------------------------------------------------------------------------
+# eq:sign_rule: brute force over both scale signs
+# --------------------------------------------------------------------------
+
+def _groups_for_sign_tests():
+    out = [w for w in lattice_groups(3, 8)]
+    out += list(random_groups(300, 32, 5))
+    out += list(random_groups(100, 128, 6))
+    return out
+
+
+@pytest.mark.parametrize("q", QS)
+def test_sign_rule_against_both_signs(q):
+    half = 1 << (q - 1)
+    for w in _groups_for_sign_tests():
+        mx, mn = float(np.max(w)), float(np.min(w))
+        sig = oracle.quantize_group(w, q, oracle.GRID_SIGNED_SYM)
+        uns = oracle.quantize_group(w, q, oracle.GRID_UNSIGNED_SYM)
+        both = {gm: oracle.quantize_group_gamma(w, q, gm) for gm in (1, -1)}
+        # the signed grid is the gamma-quantizer at its chosen sign, and the
+        # unsigned grid is the gamma = +1 quantizer (eq:signed_sym_quant)
+        assert np.array_equal(sig["c"], both[sig["gamma"]]["c"])
+        assert sig["s32"] == both[sig["gamma"]]["s32"]
+        assert np.array_equal(uns["c"], both[1]["c"]) and uns["gamma"] == 1
+        if mx == -mn:
+            assert sig["gamma"] == 1  # tie reading
+            continue
+        i, wi = dominant_outlier(w)
+        # exactly one sign represents the dominant outlier exactly
+        exact = [gm for gm in (1, -1)
+                 if F(both[gm]["s32"]) * both[gm]["c"][i] == F(wi)]
+        assert exact == [sig["gamma"]]
+        assert sig["c"][i] == -half
+        # and it is -sign(w_i*)
+        assert sig["gamma"] == (-1 if wi > 0 else 1)
+
+
+@pytest.mark.parametrize("q", QS)
+def test_unsigned_equals_signed_when_outlier_negative(q):
+    W = random_groups(400, 32, 21)
+    n_neg = 0
+    for w in W:
+        if float(np.max(w)) < -float(np.min(w)):
+            n_neg += 1
+            a = oracle.quantize_group(w, q, oracle.GRID_UNSIGNED_SYM)
+            b = oracle.quantize_group(w, q, oracle.GRID_SIGNED_SYM)
+            assert np.array_equal(a["u"], b["u"]) and a["s16"] == b["s16"]
+    assert n_neg > 50
+
+
+# --------------------------------------------------------------------------
+# def:clipped-set, the structural properties, lem:error-separability,
+# thm:worst-case-bound and cor:optimal-sign -- in exact arithmetic
+# --------------------------------------------------------------------------
+
+def _exact_group_terms(w, q, gamma, r):
+    M = F(float(r["M"]))
+    alpha = abs(F(r["s32"]))
+    T = M * (1 - F(1, 1 << q))
+    wf = [F(float(v)) for v in w]
+    Qw = [F(r["s32"]) * c for c in r["c"]]
+    return M, alpha, T, wf, Qw
+
+
+@pytest.mark.parametrize("q", QS)
+def test_clipped_set_and_lemma_and_bound(q):
+    half = 1 << (q - 1)
+    n_checked = 0
+    for w in _groups_for_sign_tests():
+        if float(np.max(np.abs(w))) == 0:
+            continue
+        res = {gm: oracle.quantize_group_gamma(w, q, gm) for gm in (1, -1)}
+        for gm, r in res.items():
+            M, alpha, T, wf, Qw = _exact_group_terms(w, q, gm, r)
+            midpoint = any(is_midpoint(x / alpha) for x in wf)
+            C = {j for j, cp in enumerate(r["c_pre"]) if cp == half}
+            Cother = {j for j, cp in enumerate(r["c_pre"]) if cp == -half}
+            assert r["n_self"] == len(C) and r["n_other"] == len(Cother)
+            # the other sign's clipped set is this sign's lower-tail set
+            assert Cother == {j for j, cp in enumerate(res[-gm]["c_pre"]) if cp == half}
+            err = [(x - qx) ** 2 for x, qx in zip(wf, Qw)]
+            # thm:worst-case-bound, total (holds at midpoints too)
+            d = len(wf)
+            assert sum(err) <= F(1, 1 << (2 * q)) * M * M * d * (1 + 3 * F(len(C), d))
+            if midpoint:
+                continue
+            n_checked += 1
+            # def:clipped-set: C_gamma = {i : gamma w_i > M (1 - 2^-q)}
+            assert C == {j for j, x in enumerate(wf) if gm * x > T}
+            # thm:worst-case-bound, per coordinate
+            for j, e in enumerate(err):
+                if j in C:
+                    assert alpha * alpha / 4 < e <= alpha * alpha
+                else:
+                    assert e <= alpha * alpha / 4
+            # lem:error-separability: ||w - Q||^2 = E(w) + 2 alpha sum_C (gamma w_i - T)
+            E = sum((x - alpha * round(x / alpha)) ** 2 for x in wf)
+            assert sum(err) == E + 2 * alpha * sum(gm * wf[j] - T for j in C)
+        # cor:optimal-sign and rem:cardinality-margin, at gamma* of the sign rule
+        mx, mn = float(np.max(w)), float(np.min(w))
+        gs = -1 if mx > -mn else 1
+        a, b = res[gs], res[-gs]
+        margin = b["n_self"] - a["n_self"]
+        bound = lambda r: F(1, 1 << (2 * q)) * F(float(r["M"])) ** 2 * len(w) * (1 + 3 * F(r["n_self"], len(w)))
+        if margin >= 0:
+            assert bound(a) <= bound(b)
+        # structural: C_gamma* lies in {gamma* w_i > 0}
+        assert all(gs * float(w[j]) > 0 for j, cp in enumerate(a["c_pre"]) if cp == half)
+    assert n_checked > 500
+
+
+# --------------------------------------------------------------------------
+# thm:signed-asymmetric: Q(w; -alpha, 0) == Q(w; alpha, -1)
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("q", QS)
+def test_sign_flip_is_unit_zero_point_shift(q):
+    A = alphabet(q)
+    n = 0
+    groups = list(random_groups(300, 32, 5)) + list(lattice_groups(3, 8))[::7]
+    for w in groups:
+        if float(np.max(np.abs(w))) == 0:
+            continue
+        r = oracle.quantize_group_gamma(w, q, -1)
+        alpha = -F(r["s32"])
+        assert alpha > 0
+        for j, x in enumerate(w):
+            x = F(float(x))
+            if is_midpoint(x / alpha):
+                continue
+            # Q(w; alpha, -1) = alpha * (clip(round(w/alpha - 1)) + 1): the
+            # nearest point of the shifted grid alpha*(A_q + 1), by brute force
+            rhs = alpha * (nearest_index(x, alpha, alpha, A) + 1)
+            assert F(r["s32"]) * r["c"][j] == rhs
+            n += 1
+    assert n > 9000
+
+
+def test_sign_flip_integer_identity_exhaustive():
+    """-clip(-RNE(x)) == clip(RNE(x - 1)) + 1 for every non-midpoint x on a
+    fine dyadic lattice (both sides give the nearest point of A_q + 1)."""
+    for q in QS:
+        lo, hi = -(1 << (q - 1)), (1 << (q - 1)) - 1
+        for num in range(-40 * 64, 40 * 64 + 1):
+            x = F(num, 64)
+            if is_midpoint(x):
+                continue
+            lhs = -min(max(round(-x), lo), hi)
+            rhs = min(max(round(x - 1), lo), hi) + 1
+            assert lhs == rhs
+
+
+# --------------------------------------------------------------------------
+# code range, on-grid round trip
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("grid", [0, 1, 2])
+@pytest.mark.parametrize("q", QS)
+def test_code_range(q, grid):
+    W = inputs.student_t_weights(64, 4096, 99 + q)
+    codes, scales, mins, clip, flags = oracle.quantize(W, q, 32, grid, clip_counts=True)
+    assert flags == 0
+    u = np.stack([oracle.unpack_group(codes.reshape(-1, 32 * q // 8)[G], 32, q)
+                  for G in range(codes.size // (32 * q // 8))])
+    assert u.min() >= 0 and u.max() <= (1 << q) - 1
+
+
+@pytest.mark.parametrize("q", QS)
+def test_on_grid_round_trip(q):
+    rng = np.random.default_rng(3)
+    half = 1 << (q - 1)
+    for _ in range(300):
+        gamma = int(rng.choice([-1, 1]))
+        alpha = 2.0 ** int(rng.integers(-12, 4))
+        a = rng.integers(-half + 1, half, 32)
+        a[int(rng.integers(0, 32))] = -half   # the dominant outlier at -2^(q-1)
+        w = (gamma * alpha * a).astype(np.float32)
+        r = oracle.quantize_group(w, q, oracle.GRID_SIGNED_SYM)
+        assert r["gamma"] == gamma
+        assert np.array_equal(r["c"], a)
+
+
+# --------------------------------------------------------------------------
+# eq:minmax asymmetric grid
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("q", QS)
+def test_asym_codes_are_nearest_grid_points(q):
+    umax = (1 << q) - 1
+    groups = list(lattice_groups(3, 8)) + list(random_groups(200, 32, 17))
+    for w in groups:
+        r = oracle.quantize_group(w, q, oracle.GRID_ASYM)
+        mn, mx = float(np.min(w)), float(np.max(w))
+        if mx == mn:
+            assert np.all(r["u"] == 0)
+            continue
+        s = F(r["s32"])
+        assert s > 0
+        # the stored min and scale are the fp16 roundings (numpy's conversion)
+        assert r["m16"] == int(np.float16(np.float32(mn)).view(np.uint16))
+        assert r["s16"] == int(np.float16(np.float32(r["s32"])).view(np.uint16))
+        for j, x in enumerate(w):
+            d = np.float32(x) - np.float32(mn)  # the fl32(w - min) of the reading
+            u = nearest_index(F(float(d)), F(0), s, range(umax + 1))
+            assert r["u"][j] == u
+            if F(float(d)) == F(float(x)) - F(mn):  # exact subtraction
+                assert abs(F(float(x)) - (F(mn) + s * r["u"][j])) <= s / 2
+        assert r["u"][int(np.argmin(w))] == 0
+        assert r["u"][int(np.argmax(w))] == umax
+
+
+# --------------------------------------------------------------------------
+# packed layout
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("q", QS)
+@pytest.mark.parametrize("g", [8, 32, 128])
+def test_pack_layout_bitwise(q, g):
+    rng = np.random.default_rng(q * 1000 + g)
+    for _ in range(50):
+        u = rng.integers(0, 1 << q, g).astype(np.uint8)
+        b = oracle.pack_group(u, q)
+        assert b.size == g * q // 8
+        bits = np.unpackbits(b, bitorder="little")
+        if q == 4:
+            got = bits.reshape(g, 4) @ (1 << np.arange(4))
+        elif q == 2:
+            got = bits.reshape(g, 2) @ (1 << np.arange(2))
+        else:
+            lo = bits[: 2 * g].reshape(g, 2) @ (1 << np.arange(2))
+            hi = bits[2 * g:]
+            got = lo + 4 * hi
+        assert np.array_equal(got, u)
+        assert np.array_equal(oracle.unpack_group(b, g, q), u)
+
+
+def test_matrix_quantize_is_groupwise():
+    for q in QS:
+        for grid in (0, 1, 2):
+            W = random_groups(6, 256, 31 + q)
+            W = W.reshape(6, 256)
+            codes, scales, mins, clip, _ = oracle.quantize(W, q, 32, grid, clip_counts=True)
+            gb = 32 * q // 8
+            flat = W.reshape(-1, 32)
+            for G in range(flat.shape[0]):
+                r = oracle.quantize_group(flat[G], q, grid)
+                assert bytes(codes.reshape(-1, gb)[G]) == bytes(oracle.pack_group(r["u"], q))
+                assert scales.ravel()[G] == r["s16"]
+                if grid == 2:
+                    assert mins.ravel()[G] == r["m16"]
+                assert clip.reshape(-1, 2)[G, 0] == r["n_self"]
+                assert clip.reshape(-1, 2)[G, 1] == r["n_other"]
+
+
+# --------------------------------------------------------------------------
+# dequantisation and the fp64 matmul reference
+# --------------------------------------------------------------------------
+
+def _numpy_dequant(codes, scales, mins, n, k, q, g, grid):
+    gb = g * q // 8
+    u = np.stack([oracle.unpack_group(cg, g, q) for cg in codes.reshape(-1, gb)])
+    s = scales.reshape(-1, 1).view(np.float16).astype(np.float32)
+    if grid == oracle.GRID_ASYM:
+        m = mins.reshape(-1, 1).view(np.float16).astype(np.float32)
+        return (s * u.astype(np.float32) + m).reshape(n, k)
+    return (s * (u.astype(np.float32) - (1 << (q - 1)))).reshape(n, k)
+
+
+@pytest.mark.parametrize("grid", [0, 1, 2])
+@pytest.mark.parametrize("q", QS)
+def test_dequantize_matches_numpy(q, grid):
+    n, k, g = 16, 256, 32
+    W = inputs.student_t_weights(n, k, 5 + q)
+    codes, scales, mins, _, _ = oracle.quantize(W, q, g, grid)
+    got = oracle.dequantize(codes, scales, mins, n, k, q, g, grid)
+    ref = _numpy_dequant(codes, scales, mins, n, k, q, g, grid)
+    assert np.array_equal(got.view(np.uint32), ref.view(np.uint32))
+    part = oracle.dequantize(codes, scales, mins, n, k, q, g, grid, rows=(5, 3))
+    assert np.array_equal(part, got[5:8])
+
+
+def test_matmul_f64_matches_numpy():
+    rng = np.random.default_rng(0)
+    What = rng.standard_normal((40, 300)).astype(np.float32)
+    xb = inputs.normal_bf16_bits((3, 300), 1)
+    x = inputs.bf16_bits_to_f32(xb).astype(np.float64)
+    ref = x @ What.astype(np.float64).T
+    got = oracle.matmul_f64(What, xb)
+    np.testing.assert_allclose(got, ref, rtol=1e-12, atol=1e-12)
+    # a one-hot activation picks one column of the weights exactly
+    e = np.zeros((1, 300), np.float32)
+    e[0, 17] = 1.0
+    assert np.array_equal(oracle.matmul_f64(What, inputs.f32_to_bf16_bits(e))[0],
+                          What[:, 17].astype(np.float64))
+
+
+@pytest.mark.parametrize("grid", [0, 1, 2])
+def test_gemv_is_matmul_of_dequantised(grid):
+    n, k, q, g = 24, 512, 3, 32
+    W = inputs.student_t_weights(n, k, 8)
+    codes, scales, mins, _, _ = oracle.quantize(W, q, g, grid)
+    xb = inputs.normal_bf16_bits((4, k), 2)
+    y = oracle.gemv(codes, scales, mins, n, k, q, g, grid, xb)
+    What = _numpy_dequant(codes, scales, mins, n, k, q, g, grid)
+    ref = inputs.bf16_bits_to_f32(xb).astype(np.float64) @ What.astype(np.float64).T
+    np.testing.assert_allclose(y, ref, rtol=1e-12, atol=1e-12)
+
+
+# --------------------------------------------------------------------------
+# flags and extreme magnitudes
+# --------------------------------------------------------------------------
+
+def test_nonfinite_and_range_flags():
+    w = inputs.student_t_weights(1, 32, 3)[0]
+    bad = w.copy()
+    bad[5] = np.nan
+    for grid in (0, 1, 2):
+        assert oracle.quantize_group(bad, 4, grid)["flags"] & oracle.FLAG_NONFINITE
+        assert oracle.quantize_group(w, 4, grid)["flags"] == 0
+    big = (w / np.max(np.abs(w)) * 1e6).astype(np.float32)
+    assert oracle.quantize_group(big, 2, 1)["flags"] & oracle.FLAG_RANGE
+
+
+@pytest.mark.parametrize("q", QS)
+@pytest.mark.parametrize("e", [-140, -130, -100, -20, 20, 60, 100])
+def test_extreme_magnitudes_still_round_to_nearest(q, e):
+    """Subnormal and huge groups: codes stay the nearest grid points for the
+    scale the oracle used (eq:quantizer), for both signs."""
+    A = alphabet(q)
+    W = random_groups(20, 32, 1000 + e + q)
+    for w in W:
+        w = (w.astype(np.float64) * 2.0 ** e).astype(np.float32)
+        if float(np.max(np.abs(w))) == 0:
+            continue
+        for gm in (1, -1):
+            r = oracle.quantize_group_gamma(w, q, gm)
+            s = F(r["s32"])
+            if s == 0:
+                continue
+            for j in range(32):
+                assert r["c"][j] == nearest_index(F(float(w[j])), F(0), s, A)
