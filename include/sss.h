@@ -1,0 +1,186 @@
+/*
+ * sss.h -- C ABI of the GB300 (sm_103a) signed-symmetric few-bit weight
+ * library: group-wise q-bit weight quantization with a signed per-group scale
+ * and no zero point, and the decode GEMV / prefill GEMM that consume the
+ * packed codes with dequantisation fused in.
+ *
+ * Source of the operations: Colbert, Dash et al., "Signed Symmetric
+ * Quantization for Few-Bit Integers": the integer quantizer (eq:quantizer,
+ * Sec. 1), the min-max grid (eq:minmax) and absmax grid (eq:absmax) of
+ * Sec. 3, the signed symmetric family (eq:signed_sym_quant) and the signed
+ * absmax sign rule (eq:sign_rule), the direct-casting protocol (Appendix C.1)
+ * and the deployed block formats and quantized GEMM expansion (Appendix B).
+ *
+ * Conventions for every entry point:
+ *  - All tensor pointers are DEVICE pointers owned by the caller.  No entry
+ *    point allocates device memory (sss_gemm keeps a small per-device cache
+ *    of encoded tensor maps in host memory).
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream).  Every call is asynchronous on that stream; none synchronises.
+ *  - The return value reports synchronous argument checks and launch errors.
+ *    Data-dependent conditions (NaN/Inf weights, a scale that overflows
+ *    fp16, a wait that timed out) are OR-ed as SSS_FLAG_* bits into the
+ *    optional device word `dev_status` (uint32), which the caller zeroes and
+ *    reads back after synchronising.
+ *  - No C++ exception crosses the ABI.  Functions are thread-safe.
+ *
+ * Weight layout: W is row-major fp32 [n][k] (n = output features, k = input
+ * features, the quantized axis); groups are `group` consecutive elements
+ * along k, so group G = row*(k/group) + j starts at element G*group.
+ * Packed codes are stored per group, groups back to back (codes of group G
+ * start at byte G*group*q/8):
+ *   q=4: element j in byte j>>1, low nibble for even j, high for odd j;
+ *   q=2: element j in byte j>>2 at bits 2*(j&3);
+ *   q=3: a plane of group/4 bytes holding (u & 3) in the q=2 layout, then a
+ *        plane of group/8 bytes with bit (j&7) of byte (j>>3) = (u >> 2).
+ * The stored code is u = c + 2^(q-1) for the symmetric grids (c in the signed
+ * alphabet {-2^(q-1) .. 2^(q-1)-1}) and u = c in {0 .. 2^q-1} for ASYM.
+ * scales: IEEE fp16 [n][k/group], the signed scale s = gamma*alpha for the
+ * symmetric grids (Appendix B.1: "may be negative"), the step for ASYM.
+ * mins: fp16 [n][k/group], ASYM only (the stored minimum m; w^ = s*u + m).
+ */
+#ifndef SSS_H
+#define SSS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SSS_GRID_UNSIGNED_SYM = 0, /* absmax grid, s = ||w||_inf / 2^(q-1) > 0 (eq:absmax)      */
+  SSS_GRID_SIGNED_SYM = 1,   /* signed absmax, s = gamma* alpha (eq:signed_sym_quant,
+                                eq:sign_rule); gamma = +1 when max w == -min w            */
+  SSS_GRID_ASYM = 2          /* min-max grid on {0..2^q-1} (eq:minmax)                  */
+} sss_grid_t;
+
+typedef enum {
+  SSS_OK = 0,
+  SSS_E_ARG = 1,         /* a size or enum argument is out of range / NULL         */
+  SSS_E_UNSUPPORTED = 2, /* a combination this build does not implement            */
+  SSS_E_ALIGN = 3,       /* a pointer is not aligned as documented                 */
+  SSS_E_CUDA = 4,        /* a CUDA runtime/driver call or launch failed            */
+  SSS_E_WORKSPACE = 5    /* workspace too small (see sss_workspace_bytes)          */
+} sss_status_t;
+
+/* bits OR-ed into *dev_status by the kernels */
+#define SSS_FLAG_NONFINITE 0x1u /* a weight group contains NaN or +-Inf; that group's
+                                   codes/scale are placeholders (u = 2^(q-1) and s = +0
+                                   for symmetric grids, u = 0 and s = +0 for ASYM)     */
+#define SSS_FLAG_RANGE 0x2u     /* a stored fp16 scale or min is infinite (|s| >= 65520),
+                                   or the fp32 ASYM step overflowed (codes then 0)     */
+#define SSS_FLAG_TIMEOUT 0x4u   /* a bounded pipeline wait in sss_gemm expired; the
+                                   output is incomplete                               */
+
+typedef enum { SSS_OUT_F32 = 0, SSS_OUT_F16 = 1, SSS_OUT_BF16 = 2 } sss_dtype_t;
+
+/* A packed weight tensor.  Plain descriptor; the library never frees it. */
+typedef struct {
+  int64_t n;         /* rows (output features), >= 0                                */
+  int64_t k;         /* columns (input features), multiple of `group`             */
+  int32_t q;         /* bits per code: 2, 3 or 4                                   */
+  int32_t group;     /* group size along k: 32, 64 or 128                          */
+  int32_t grid;      /* sss_grid_t                                                 */
+  int32_t reserved;  /* must be 0                                                  */
+  uint8_t* codes;    /* [n][k*q/8] bytes, layout above                             */
+  uint16_t* scales;  /* [n][k/group] fp16                                          */
+  uint16_t* mins;    /* [n][k/group] fp16 for SSS_GRID_ASYM, else ignored (NULL)   */
+} sss_qtensor_t;
+
+/* Bytes of packed codes for an [n][k] tensor at q bits: n*k*q/8. */
+size_t sss_codes_bytes(int64_t n, int64_t k, int32_t q);
+
+/* Human-readable name of a status code (static storage). */
+const char* sss_status_string(sss_status_t status);
+
+/* Text of the last CUDA error seen by this thread inside the library
+ * (static thread-local storage; "" if none). */
+const char* sss_last_error(void);
+
+/*
+ * sss_quantize -- direct casting of an fp32 weight matrix (Appendix C.1):
+ * for every group, M = ||w||_inf, the grid's scale (eq:absmax; eq:sign_rule
+ * for SIGNED: gamma* = -sign(w_i*), so the dominant outlier lands exactly on
+ * the code -2^(q-1); eq:minmax for ASYM), codes c = clip(RNE(w/s)) of the
+ * exact quotient (ties to even), packed as above, and the fp16 scale (and
+ * min).  Bit-exact with the reference definition.
+ *
+ *   w           [in]  device fp32 [n][k], 16-byte aligned, row-major contiguous.
+ *   out         [in]  descriptor of the outputs (n, k, q, group, grid and the
+ *                     device buffers codes, scales, mins); not retained.
+ *   clip_counts [out] nullable device uint8 [n][k/group][2]: for symmetric
+ *                     grids {|C_gamma|, |C_-gamma|} (def:clipped-set): the
+ *                     number of pre-clip codes equal to +2^(q-1) and to
+ *                     -2^(q-1); for ASYM {0, 0}.
+ *   dev_status  [out] nullable device uint32; SSS_FLAG_NONFINITE/RANGE OR-ed.
+ * Errors: SSS_E_ARG (q, group, grid, k % group, NULL buffers), SSS_E_ALIGN
+ * (w not 16-byte aligned), SSS_E_CUDA.  n == 0 is a no-op.
+ */
+sss_status_t sss_quantize(const float* w, const sss_qtensor_t* out,
+                          uint8_t* clip_counts, uint32_t* dev_status,
+                          void* stream);
+
+/*
+ * sss_dequantize -- w^ = f16(s)*c (symmetric; exact in fp32) or
+ * w^ = fl32(fl32(f16(s)*u) + f16(m)) (ASYM), the value eq:quantizer assigns
+ * to each weight, written as [n][k] in out_dtype (fp16/bf16 outputs are the
+ * round-to-nearest-even of the fp32 value).
+ *   qt   [in]  packed tensor (device buffers).
+ *   out  [out] device [n][k] of sss_dtype_t out_dtype, 16-byte aligned.
+ * Errors: SSS_E_ARG, SSS_E_ALIGN, SSS_E_CUDA.
+ */
+sss_status_t sss_dequantize(const sss_qtensor_t* qt, void* out,
+                            int32_t out_dtype, void* stream);
+
+/*
+ * sss_gemv -- decode GEMV y[b][r] = sum_k w^[r][k] * x[b][k] with the
+ * dequantisation fused (Appendix B.3: y = sum_b s * (integer dot) for the
+ * symmetric formats, plus the row-sum term sum_b m * sum_{k in b} x for
+ * ASYM).  fp32 accumulation; deterministic (no atomics).
+ *   qt        [in]  packed tensor; codes 16-byte aligned, scales/mins 4-byte
+ *                   aligned.
+ *   x_bf16    [in]  device bf16 [batch][k], 16-byte aligned.
+ *   batch     [in]  1..16.
+ *   y         [out] device fp32 [batch][n].
+ *   workspace [in]  device scratch of ws_bytes >= sss_workspace_bytes(qt,
+ *                   batch, SSS_OP_GEMV) bytes, 16-byte aligned, or NULL when
+ *                   that size is 0.  Its contents on entry are ignored.
+ *   dev_status [out] nullable; unused by the GEMV (reserved).
+ * Errors: SSS_E_ARG, SSS_E_ALIGN, SSS_E_WORKSPACE, SSS_E_CUDA.
+ */
+sss_status_t sss_gemv(const sss_qtensor_t* qt, const uint16_t* x_bf16,
+                      int32_t batch, float* y, void* workspace,
+                      size_t ws_bytes, uint32_t* dev_status, void* stream);
+
+/*
+ * sss_gemm -- prefill GEMM Y[m][r] = sum_k w^[r][k] * X[m][k] (Appendix B.3,
+ * "compute-bound phase dominated by matrix multiplications"), dequantising
+ * weight tiles on chip and accumulating on the tcgen05 tensor cores in fp32
+ * (tensor memory).  Tile operands are fp16: w^ rounded to fp16 and X
+ * converted from bf16 (exact for 2^-17 <= |x| <= 65504).
+ *   qt        [in]  packed tensor, symmetric grids or ASYM; k % 64 == 0;
+ *                   codes 16-byte aligned.
+ *   x_bf16    [in]  device bf16 [m][k], 16-byte aligned.
+ *   m         [in]  >= 0 tokens.
+ *   y         [out] device fp32 [m][n], 16-byte aligned, n % 4 == 0.
+ *   workspace [in]  as for sss_gemv with SSS_OP_GEMM.
+ *   dev_status [out] nullable; SSS_FLAG_TIMEOUT if a bounded wait expired.
+ * Errors: SSS_E_ARG, SSS_E_ALIGN, SSS_E_UNSUPPORTED, SSS_E_WORKSPACE, SSS_E_CUDA.
+ */
+sss_status_t sss_gemm(const sss_qtensor_t* qt, const uint16_t* x_bf16,
+                      int64_t m, float* y, void* workspace, size_t ws_bytes,
+                      uint32_t* dev_status, void* stream);
+
+#define SSS_OP_GEMV 0
+#define SSS_OP_GEMM 1
+/* Workspace bytes sss_gemv (op SSS_OP_GEMV, m_or_batch = batch) or sss_gemm
+ * (op SSS_OP_GEMM, m_or_batch = m) needs for this tensor; 0 if none. */
+size_t sss_workspace_bytes(const sss_qtensor_t* qt, int64_t m_or_batch,
+                           int32_t op);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SSS_H */

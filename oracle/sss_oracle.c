@@ -163,6 +163,10 @@ static int32_t quantize_group_asym(const float* w, int32_t g, int32_t q,
   orc_group_t r;
   memset(&r, 0, sizeof r);
   r.flags = scan_group(w, g, &r.mx, &r.mn);
+  /* reading: a zero minimum is stored as +0 (the sign of zero of a group
+   * mixing +0 and -0 is otherwise an artefact of the scan order) */
+  if (r.mn == 0.0f) r.mn = 0.0f;
+  if (r.mx == 0.0f) r.mx = 0.0f;
   r.M = (r.mx > -r.mn) ? r.mx : -r.mn;
   r.gamma = 0;
   const int32_t umax = (1 << q) - 1;

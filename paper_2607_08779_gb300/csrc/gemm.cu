@@ -1,0 +1,552 @@
+// gemm.cu -- prefill GEMM over packed q-bit codes on the 5th-generation
+// tensor cores (sm_103a: tcgen05 + tensor memory + TMA).
+//
+// Y[m][r] = sum_k w^[r][k] X[m][k]; the prefill phase is "a compute-bound
+// phase dominated by matrix multiplications" (Appendix B.2), and the
+// symmetric formats compute only the integer-code GEMM term of the expansion
+// in Appendix B.3 (the min-max grid adds the per-block minimum).
+//
+// Precision: the dequantised weight s*c is rounded to fp16 (<= 2^-11
+// relative, where bf16 would give 2^-8 and miss the 1e-3 output gate) and
+// the bf16 activations are converted to fp16 (exact for 2^-17 <= |x| <=
+// 65504).  tcgen05.mma kind::f16 takes both operands in fp16 and accumulates
+// in fp32 in tensor memory.
+//
+// Structure (one CTA per 128-row x BN-token output tile, 6 warps):
+//   warp 0     TMA producer for the fp16 activation tile (128B swizzle) and
+//              owner of the tensor-memory allocation;
+//   warp 1     a single elected thread issues tcgen05.mma (M=128, N=BN,
+//              K=16 per instruction, 4 per 64-wide k-block) and commits to
+//              the stage's "empty" barrier;
+//   warps 2-5  dequantise: each thread owns one weight row of the tile,
+//              loads that row's codes and scales for the k-block, forms fp16
+//              s*c in natural k order and stores it with the 128B swizzle the
+//              shared-memory descriptor expects; after the last k-block the
+//              same warps drain the fp32 accumulator with tcgen05.ld and store
+//              Y (for a fixed token, a warp writes 32 consecutive floats).
+// Every mbarrier wait is bounded (about one second of global time); on
+// expiry the CTA raises SSS_FLAG_TIMEOUT, all roles leave their loops, and
+// the tensor memory is still released.
+#include <cuda.h>
+
+#include <algorithm>
+#include <mutex>
+
+#include "sss_internal.cuh"
+
+namespace sss {
+namespace {
+
+constexpr int kBM = 128;            // weight rows per tile (MMA M)
+constexpr int kBK = 64;             // k per stage (128 bytes of fp16)
+constexpr int kThreads = 192;
+constexpr uint64_t kWaitNs = 1000000000ull;  // bounded waits: 1 s
+
+// ---------------------------------------------------------------------------
+// PTX wrappers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait on a phase parity.  Returns false when the wait gave up,
+// either on its own time limit or because another role raised *abort.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity,
+                                          volatile int* abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 255u) == 0) {
+      if (*abort) return false;
+      if (global_ns() - t0 > kWaitNs) {
+        *abort = 1;
+        return false;
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void tma_load_2d(const CUtensorMap* map, uint64_t* bar, void* dst,
+                                            int c0, int c1) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1)
+      : "memory");
+}
+
+// tcgen05 shared-memory matrix descriptor: K-major operand, 128-byte swizzle,
+// 8-row swizzle atoms 1024 bytes apart (stride byte offset), descriptor
+// version 1 at bit 46.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);          // start address
+  d |= static_cast<uint64_t>(1) << 16;                           // LBO (unused for SW128 K-major)
+  d |= static_cast<uint64_t>(1024 >> 4) << 32;                    // SBO: 1024 B
+  d |= static_cast<uint64_t>(1) << 46;                           // version
+  d |= static_cast<uint64_t>(2) << 61;                           // 128B swizzle
+  return d;
+}
+
+// Instruction descriptor, kind::f16: D fp32, A and B fp16, both K-major.
+__host__ __device__ constexpr uint32_t make_idesc(int M, int N) {
+  return (1u << 4)                                    // D format: F32
+         | (0u << 7) | (0u << 10)                     // A, B format: F16
+         | (static_cast<uint32_t>(N >> 3) << 17)      // N / 8
+         | (static_cast<uint32_t>(M >> 4) << 24);     // M / 16
+}
+
+__device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+        "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+        "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// ---------------------------------------------------------------------------
+// Dequantisation of 32 codes of one row into 16 natural-order fp16 pairs.
+// ---------------------------------------------------------------------------
+
+// PRMT selector: result = [a.byte_i, 0, b.byte_i, 0]; the zero bytes use the
+// sign-replicate mode on a byte whose top bit is clear.
+__device__ __forceinline__ uint32_t pair_bytes(uint32_t a, uint32_t b, int i) {
+  const uint32_t sel = static_cast<uint32_t>(i) | (static_cast<uint32_t>(8 + i) << 4) |
+                       (static_cast<uint32_t>(4 + i) << 8) |
+                       (static_cast<uint32_t>(12 + i) << 12);
+  uint32_t r;
+  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(r) : "r"(a), "r"(b), "r"(sel));
+  return r;
+}
+
+// u pairs (natural order: element 2p in the low half, 2p+1 in the high half)
+// of a 32-code sub-chunk, as 16-bit integers.
+template <int Q>
+__device__ __forceinline__ void code_pairs(const uint32_t* w, uint32_t (&u)[16]) {
+  if constexpr (Q == 4) {
+#pragma unroll
+    for (int wi = 0; wi < 4; ++wi) {
+      const uint32_t ev = w[wi] & 0x0F0F0F0Fu, od = (w[wi] >> 4) & 0x0F0F0F0Fu;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) u[4 * wi + i] = pair_bytes(ev, od, i);
+    }
+  } else {
+#pragma unroll
+    for (int wi = 0; wi < 2; ++wi) {
+      const uint32_t a = w[wi] & 0x03030303u, b = (w[wi] >> 2) & 0x03030303u;
+      const uint32_t c = (w[wi] >> 4) & 0x03030303u, d = (w[wi] >> 6) & 0x03030303u;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        u[8 * wi + 2 * i] = pair_bytes(a, b, i);
+        u[8 * wi + 2 * i + 1] = pair_bytes(c, d, i);
+      }
+    }
+    if constexpr (Q == 3) {
+      const uint32_t hi = w[2];
+#pragma unroll
+      for (int p = 0; p < 16; ++p) {
+        const uint32_t v = (hi >> (2 * p)) & 3u;
+        u[p] |= ((v & 1u) << 2) | ((v & 2u) << 17);  // + 4*hi bit, both halves
+      }
+    }
+  }
+}
+
+template <int Q>
+__device__ __forceinline__ void load_sub32(const uint8_t* __restrict__ row, int64_t grp, int sc,
+                                           int G, bool valid, uint32_t* w) {
+  if constexpr (Q == 4) {
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (valid) v = __ldcs(reinterpret_cast<const uint4*>(row + grp * (G / 2) + sc * 16));
+    w[0] = v.x; w[1] = v.y; w[2] = v.z; w[3] = v.w;
+  } else if constexpr (Q == 2) {
+    uint2 v = make_uint2(0, 0);
+    if (valid) v = __ldcs(reinterpret_cast<const uint2*>(row + grp * (G / 4) + sc * 8));
+    w[0] = v.x; w[1] = v.y;
+  } else {
+    w[0] = w[1] = w[2] = 0;
+    if (valid) {
+      const uint32_t* base = reinterpret_cast<const uint32_t*>(row + grp * (3 * G / 8));
+      w[0] = __ldcs(base + 2 * sc);
+      w[1] = __ldcs(base + 2 * sc + 1);
+      w[2] = __ldcs(base + G / 16 + sc);
+    }
+  }
+}
+
+struct GemmArgs {
+  const uint8_t* codes;
+  const uint16_t* scales;
+  const uint16_t* mins;
+  float* y;
+  uint32_t* status;
+  int64_t m, n, k;
+  int G;
+};
+
+template <int BN, int STAGES>
+struct Smem {
+  static constexpr int A_BYTES = kBM * kBK * 2;   // 16 KB
+  static constexpr int B_BYTES = BN * kBK * 2;    // 16 or 32 KB
+  static constexpr int STAGE = A_BYTES + B_BYTES;
+  static constexpr int BAR_OFF = STAGES * STAGE;  // after the 1024-aligned stages
+  static constexpr int TOTAL = BAR_OFF + (3 * STAGES + 1) * 8 + 16 + 1024;  // + align slack
+};
+
+template <int Q, bool ASYM, int BN, int STAGES>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_kernel(const __grid_constant__ CUtensorMap xmap, const GemmArgs a) {
+  using S = Smem<BN, STAGES>;
+  extern __shared__ unsigned char smem_raw[];
+  // 1024-byte alignment for the swizzle atoms
+  unsigned char* smem = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint64_t* full_a = reinterpret_cast<uint64_t*>(smem + S::BAR_OFF);
+  uint64_t* full_b = full_a + STAGES;
+  uint64_t* empty = full_b + STAGES;
+  uint64_t* done = empty + STAGES;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int64_t n0 = static_cast<int64_t>(blockIdx.x) * kBM;
+  const int64_t m0 = static_cast<int64_t>(blockIdx.y) * BN;
+  const int nkb = static_cast<int>(a.k / kBK);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full_a[s], 4);
+      mbar_init(&full_b[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(done, 1);
+    *abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tmem_slot)),
+                 "r"(BN)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ---------------- TMA producer: activation tiles ----------------
+    if (lane == 0) {
+      int issued = 0;
+      for (int kb = 0; kb < nkb; ++kb) {
+        const int s = kb % STAGES;
+        const uint32_t ph = static_cast<uint32_t>(kb / STAGES) & 1u;
+        if (!mbar_wait(&empty[s], ph ^ 1u, abort)) break;
+        unsigned char* sb = smem + s * S::STAGE + S::A_BYTES;
+        mbar_arrive_expect_tx(&full_b[s], S::B_BYTES);
+        tma_load_2d(&xmap, &full_b[s], sb, kb * kBK, static_cast<int>(m0));
+        issued = kb + 1;
+      }
+      if (*abort) {
+        // let this CTA's copies still in flight land before the CTA exits
+        int drain = 0;
+        for (int kb = std::max(0, issued - STAGES); kb < issued; ++kb)
+          (void)mbar_wait(&full_b[kb % STAGES], static_cast<uint32_t>(kb / STAGES) & 1u, &drain);
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      constexpr uint32_t idesc = make_idesc(kBM, BN);
+      for (int kb = 0; kb < nkb; ++kb) {
+        const int s = kb % STAGES;
+        const uint32_t ph = static_cast<uint32_t>(kb / STAGES) & 1u;
+        if (!mbar_wait(&full_a[s], ph, abort)) break;
+        if (!mbar_wait(&full_b[s], ph, abort)) break;
+        tc_fence_after();
+        const uint32_t sa = smem_u32(smem + s * S::STAGE);
+        const uint32_t sb = sa + S::A_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < kBK / 16; ++kk) {
+          // advance 16 fp16 = 32 bytes along k inside the swizzled rows
+          umma_f16(tmem, sw128_desc(sa + kk * 32), sw128_desc(sb + kk * 32), idesc,
+                   (kb | kk) != 0 ? 1u : 0u);
+        }
+        umma_commit(&empty[s]);  // frees the stage once these MMAs complete
+      }
+      umma_commit(done);
+    }
+  } else {
+    // ---------------- dequantise, then epilogue ----------------
+    const int i = threadIdx.x - 64;  // 0..127: the tile row this thread owns
+    const int64_t r = n0 + i;
+    const bool rok = r < a.n;
+    const int64_t nG = a.k / a.G;
+    const uint8_t* rowp = a.codes + (rok ? r : 0) * (a.k * Q / 8);
+    const int sw = i & 7;  // swizzle phase of this row
+    bool ok = true;
+    for (int kb = 0; kb < nkb && ok; ++kb) {
+      const int s = kb % STAGES;
+      const uint32_t ph = static_cast<uint32_t>(kb / STAGES) & 1u;
+      if (!mbar_wait(&empty[s], ph ^ 1u, abort)) {
+        ok = false;
+        break;
+      }
+      unsigned char* arow = smem + s * S::STAGE + (i >> 3) * 1024 + sw * 128;
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {  // two 32-code sub-chunks per 64-wide k-block
+        const int64_t kc = static_cast<int64_t>(kb) * kBK + 32 * j;
+        const int64_t grp = kc / a.G;
+        const int sc = static_cast<int>((kc % a.G) / 32);
+        uint32_t w[4];
+        load_sub32<Q>(rowp, grp, sc, a.G, rok, w);
+        __half2 s2 = __float2half2_rn(0.f), m2 = __float2half2_rn(0.f);
+        if (rok) {
+          const __half sh = __ushort_as_half(a.scales[r * nG + grp]);
+          s2 = __halves2half2(sh, sh);
+          if constexpr (ASYM) {
+            const __half mh = __ushort_as_half(a.mins[r * nG + grp]);
+            m2 = __halves2half2(mh, mh);
+          }
+        }
+        uint32_t u[16];
+        code_pairs<Q>(w, u);
+        uint32_t out[16];
+#pragma unroll
+        for (int p = 0; p < 16; ++p) {
+          // 1024 + u as fp16, minus 1024 (+ 2^(q-1) for symmetric codes): exact
+          const uint32_t mag = u[p] | 0x64006400u;
+          __half2 hv = *reinterpret_cast<const __half2*>(&mag);
+          const __half2 bias = ASYM ? __float2half2_rn(1024.f)
+                                    : __float2half2_rn(static_cast<float>(1024 + (1 << (Q - 1))));
+          hv = __hsub2(hv, bias);                                  // c (or u) exactly
+          hv = ASYM ? __hfma2(hv, s2, m2) : __hmul2(hv, s2);       // RN16(s*c) / RN16(s*u+m)
+          out[p] = *reinterpret_cast<const uint32_t*>(&hv);
+        }
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) {  // four 16-byte chunks of 8 elements
+          const int chunk = 4 * j + cc;
+          uint4 v = make_uint4(out[4 * cc], out[4 * cc + 1], out[4 * cc + 2], out[4 * cc + 3]);
+          *reinterpret_cast<uint4*>(arow + ((chunk ^ sw) << 4)) = v;
+        }
+      }
+      fence_proxy_async_smem();  // generic-proxy stores -> visible to the tensor core
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&full_a[s]);
+    }
+    // ---------------- epilogue ----------------
+    if (ok && mbar_wait(done, 0, abort)) {
+      tc_fence_after();
+      const int sub = warp & 3;  // tensor-memory lane quarter this warp may access
+      const int row_local = sub * 32 + lane;
+      const int64_t rr = n0 + row_local;
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 32) {
+        uint32_t v[32];
+        tmem_ld32(tmem + (static_cast<uint32_t>(sub * 32) << 16) + c0, v);
+        if (rr < a.n) {
+#pragma unroll
+          for (int c = 0; c < 32; ++c) {
+            const int64_t mm = m0 + c0 + c;
+            if (mm < a.m) a.y[mm * a.n + rr] = __uint_as_float(v[c]);
+          }
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (*abort && threadIdx.x == 0 && a.status != nullptr) atomicOr(a.status, SSS_FLAG_TIMEOUT);
+  if (warp == 0) {
+    tc_fence_after();
+    if (*abort) {  // MMAs still in flight must retire before the TMEM is released
+      int drain = 0;
+      (void)mbar_wait(done, 0, &drain);
+    }
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(BN)
+                 : "memory");
+  }
+}
+
+// bf16 -> fp16 activation conversion (round to nearest even)
+__global__ void __launch_bounds__(256)
+    bf16_to_f16_kernel(const uint16_t* __restrict__ x, __half* __restrict__ y, int64_t nvec) {
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec;
+       i += stride) {
+    const uint4 v = __ldcs(reinterpret_cast<const uint4*>(x) + i);
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float lo = __uint_as_float(w[e] << 16);
+      const float hi = __uint_as_float(w[e] & 0xFFFF0000u);
+      __half2 h = __floats2half2_rn(lo, hi);
+      o[e] = *reinterpret_cast<uint32_t*>(&h);
+    }
+    reinterpret_cast<uint4*>(y)[i] = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static std::once_flag once;
+  static EncodeTiledFn fn = nullptr;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+size_t x16_bytes(int64_t m, int64_t k) {
+  return (static_cast<size_t>(m) * static_cast<size_t>(k) * 2 + 255) / 256 * 256;
+}
+
+template <int Q, bool ASYM, int BN>
+cudaError_t run_gemm(const sss_qtensor_t& t, const __half* x16, int64_t m, float* y,
+                     uint32_t* status, cudaStream_t stream) {
+  constexpr int STAGES = (BN == 256) ? 4 : 6;
+  using S = Smem<BN, STAGES>;
+  EncodeTiledFn enc = encode_fn();
+  if (enc == nullptr) return cudaErrorNotSupported;
+  CUtensorMap map;
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(t.k), static_cast<cuuint64_t>(m)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(t.k) * 2};
+  const cuuint32_t box[2] = {kBK, BN};
+  const cuuint32_t estr[2] = {1, 1};
+  CUresult cr = enc(&map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<__half*>(x16), dims,
+                    strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
+  auto kern = gemm_kernel<Q, ASYM, BN, STAGES>;
+  cudaError_t e =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::TOTAL);
+  if (e != cudaSuccess) return e;
+  GemmArgs a;
+  a.codes = t.codes;
+  a.scales = t.scales;
+  a.mins = t.mins;
+  a.y = y;
+  a.status = status;
+  a.m = m;
+  a.n = t.n;
+  a.k = t.k;
+  a.G = t.group;
+  dim3 grid(static_cast<unsigned>((t.n + kBM - 1) / kBM), static_cast<unsigned>((m + BN - 1) / BN));
+  kern<<<grid, kThreads, S::TOTAL, stream>>>(map, a);
+  return cudaGetLastError();
+}
+
+template <int Q, bool ASYM>
+cudaError_t gemm_bn(const sss_qtensor_t& t, const __half* x16, int64_t m, float* y,
+                    uint32_t* status, cudaStream_t stream) {
+  if (m <= 1024) return run_gemm<Q, ASYM, 128>(t, x16, m, y, status, stream);
+  return run_gemm<Q, ASYM, 256>(t, x16, m, y, status, stream);
+}
+
+template <int Q>
+cudaError_t gemm_grid(const sss_qtensor_t& t, const __half* x16, int64_t m, float* y,
+                      uint32_t* status, cudaStream_t stream) {
+  if (t.grid == SSS_GRID_ASYM) return gemm_bn<Q, true>(t, x16, m, y, status, stream);
+  return gemm_bn<Q, false>(t, x16, m, y, status, stream);
+}
+
+}  // namespace
+
+size_t gemm_workspace_bytes(const sss_qtensor_t& t, int64_t m) { return x16_bytes(m, t.k); }
+
+cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m, float* y,
+                        void* workspace, uint32_t* status, cudaStream_t stream) {
+  __half* x16 = static_cast<__half*>(workspace);
+  const int64_t nvec = m * t.k / 8;
+  const int grid = static_cast<int>(std::min<int64_t>((nvec + 255) / 256,
+                                                      static_cast<int64_t>(device_sm_count()) * 8));
+  bf16_to_f16_kernel<<<std::max(grid, 1), 256, 0, stream>>>(x, x16, nvec);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  switch (t.q) {
+    case 2: return gemm_grid<2>(t, x16, m, y, status, stream);
+    case 3: return gemm_grid<3>(t, x16, m, y, status, stream);
+    case 4: return gemm_grid<4>(t, x16, m, y, status, stream);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace sss

@@ -1,0 +1,178 @@
+// sss_api.cu -- the C ABI declared in include/sss.h: synchronous argument
+// validation, dispatch to the kernels' launchers, and error mapping.  No
+// entry point allocates device memory.
+#include <mutex>
+#include <stdio.h>
+#include <string.h>
+
+#include "sss_internal.cuh"
+
+namespace sss {
+
+namespace {
+thread_local char g_last_error[256] = "";
+
+void set_error(const char* what, cudaError_t e) {
+  snprintf(g_last_error, sizeof g_last_error, "%s: %s (%d)", what,
+           cudaGetErrorString(e), static_cast<int>(e));
+}
+
+bool aligned(const void* p, size_t a) {
+  return (reinterpret_cast<uintptr_t>(p) % a) == 0;
+}
+
+sss_status_t check_tensor(const sss_qtensor_t* t) {
+  if (t == nullptr) return SSS_E_ARG;
+  if (t->q < 2 || t->q > 4) return SSS_E_ARG;
+  if (t->group != 32 && t->group != 64 && t->group != 128) return SSS_E_ARG;
+  if (t->grid < SSS_GRID_UNSIGNED_SYM || t->grid > SSS_GRID_ASYM) return SSS_E_ARG;
+  if (t->reserved != 0) return SSS_E_ARG;
+  if (t->n < 0 || t->k < 0) return SSS_E_ARG;
+  if (t->k % t->group != 0) return SSS_E_ARG;
+  if (t->n > 0 && t->k > 0) {
+    if (t->codes == nullptr || t->scales == nullptr) return SSS_E_ARG;
+    if (t->grid == SSS_GRID_ASYM && t->mins == nullptr) return SSS_E_ARG;
+  }
+  return SSS_OK;
+}
+
+sss_status_t finish(const char* what, cudaError_t e) {
+  if (e == cudaSuccess) return SSS_OK;
+  if (e == cudaErrorNotSupported) {
+    set_error(what, e);
+    return SSS_E_UNSUPPORTED;
+  }
+  set_error(what, e);
+  return SSS_E_CUDA;
+}
+
+}  // namespace
+
+int device_sm_count() {
+  static std::mutex mu;
+  static int cache[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  std::lock_guard<std::mutex> lock(mu);
+  if (cache[dev] == 0) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0)
+      v = 148;
+    cache[dev] = v;
+  }
+  return cache[dev];
+}
+
+}  // namespace sss
+
+using namespace sss;
+
+extern "C" {
+
+size_t sss_codes_bytes(int64_t n, int64_t k, int32_t q) {
+  if (n < 0 || k < 0 || q < 2 || q > 4) return 0;
+  return static_cast<size_t>(n) * static_cast<size_t>(k) * static_cast<size_t>(q) / 8;
+}
+
+const char* sss_status_string(sss_status_t s) {
+  switch (s) {
+    case SSS_OK: return "SSS_OK";
+    case SSS_E_ARG: return "SSS_E_ARG: invalid argument";
+    case SSS_E_UNSUPPORTED: return "SSS_E_UNSUPPORTED: unsupported combination";
+    case SSS_E_ALIGN: return "SSS_E_ALIGN: misaligned pointer";
+    case SSS_E_CUDA: return "SSS_E_CUDA: CUDA error";
+    case SSS_E_WORKSPACE: return "SSS_E_WORKSPACE: workspace too small";
+  }
+  return "unknown sss_status_t";
+}
+
+const char* sss_last_error(void) { return g_last_error; }
+
+sss_status_t sss_quantize(const float* w, const sss_qtensor_t* out,
+                          uint8_t* clip_counts, uint32_t* dev_status,
+                          void* stream) {
+  sss_status_t st = check_tensor(out);
+  if (st != SSS_OK) return st;
+  if (out->n == 0 || out->k == 0) return SSS_OK;
+  if (w == nullptr) return SSS_E_ARG;
+  if (!aligned(w, 16)) return SSS_E_ALIGN;
+  if (!aligned(out->scales, 2) || (out->mins && !aligned(out->mins, 2))) return SSS_E_ALIGN;
+  if (out->q == 4 && !aligned(out->codes, 2)) return SSS_E_ALIGN;
+  if (dev_status && !aligned(dev_status, 4)) return SSS_E_ALIGN;
+  return finish("sss_quantize",
+                launch_quantize(w, *out, clip_counts, dev_status,
+                                static_cast<cudaStream_t>(stream)));
+}
+
+sss_status_t sss_dequantize(const sss_qtensor_t* qt, void* out, int32_t out_dtype,
+                            void* stream) {
+  sss_status_t st = check_tensor(qt);
+  if (st != SSS_OK) return st;
+  if (out_dtype < SSS_OUT_F32 || out_dtype > SSS_OUT_BF16) return SSS_E_ARG;
+  if (qt->n == 0 || qt->k == 0) return SSS_OK;
+  if (out == nullptr) return SSS_E_ARG;
+  if (!aligned(out, 16)) return SSS_E_ALIGN;
+  if (!aligned(qt->codes, 4) || !aligned(qt->scales, 2) || (qt->mins && !aligned(qt->mins, 2)))
+    return SSS_E_ALIGN;
+  return finish("sss_dequantize",
+                launch_dequantize(*qt, out, out_dtype, static_cast<cudaStream_t>(stream)));
+}
+
+size_t sss_workspace_bytes(const sss_qtensor_t* qt, int64_t m_or_batch, int32_t op) {
+  if (check_tensor(qt) != SSS_OK || m_or_batch < 0) return 0;
+  if (op == SSS_OP_GEMV) return gemv_workspace_bytes(*qt, static_cast<int>(m_or_batch));
+  if (op == SSS_OP_GEMM) return gemm_workspace_bytes(*qt, m_or_batch);
+  return 0;
+}
+
+sss_status_t sss_gemv(const sss_qtensor_t* qt, const uint16_t* x_bf16, int32_t batch,
+                      float* y, void* workspace, size_t ws_bytes,
+                      uint32_t* dev_status, void* stream) {
+  (void)dev_status;
+  sss_status_t st = check_tensor(qt);
+  if (st != SSS_OK) return st;
+  if (batch < 1 || batch > 16) return SSS_E_ARG;
+  if (qt->n == 0) return SSS_OK;
+  if (x_bf16 == nullptr || y == nullptr) return SSS_E_ARG;
+  if (qt->k > 0 && (!aligned(qt->codes, 16) || !aligned(x_bf16, 16) ||
+                    !aligned(qt->scales, 2) || (qt->mins && !aligned(qt->mins, 2))))
+    return SSS_E_ALIGN;
+  if (!aligned(y, 4)) return SSS_E_ALIGN;
+  const size_t need = gemv_workspace_bytes(*qt, batch);
+  if (need > 0 && (workspace == nullptr || ws_bytes < need)) return SSS_E_WORKSPACE;
+  if (qt->k == 0) {  // empty reduction: y = 0
+    return finish("sss_gemv",
+                  cudaMemsetAsync(y, 0, sizeof(float) * static_cast<size_t>(batch) * qt->n,
+                                  static_cast<cudaStream_t>(stream)));
+  }
+  return finish("sss_gemv", launch_gemv(*qt, x_bf16, batch, y, workspace,
+                                        static_cast<cudaStream_t>(stream)));
+}
+
+sss_status_t sss_gemm(const sss_qtensor_t* qt, const uint16_t* x_bf16, int64_t m,
+                      float* y, void* workspace, size_t ws_bytes,
+                      uint32_t* dev_status, void* stream) {
+  sss_status_t st = check_tensor(qt);
+  if (st != SSS_OK) return st;
+  if (m < 0) return SSS_E_ARG;
+  if (m == 0 || qt->n == 0) return SSS_OK;
+  if (x_bf16 == nullptr || y == nullptr) return SSS_E_ARG;
+  if (qt->k % 64 != 0) return SSS_E_UNSUPPORTED;
+  if (qt->n % 4 != 0) return SSS_E_UNSUPPORTED;
+  if (!aligned(qt->codes, 16) || !aligned(x_bf16, 16) || !aligned(y, 16) ||
+      !aligned(qt->scales, 2) || (qt->mins && !aligned(qt->mins, 2)))
+    return SSS_E_ALIGN;
+  if (dev_status && !aligned(dev_status, 4)) return SSS_E_ALIGN;
+  const size_t need = gemm_workspace_bytes(*qt, m);
+  if (need > 0 && (workspace == nullptr || ws_bytes < need)) return SSS_E_WORKSPACE;
+  if (workspace != nullptr && !aligned(workspace, 16)) return SSS_E_ALIGN;
+  if (qt->k == 0) {
+    return finish("sss_gemm",
+                  cudaMemsetAsync(y, 0, sizeof(float) * static_cast<size_t>(m) * qt->n,
+                                  static_cast<cudaStream_t>(stream)));
+  }
+  return finish("sss_gemm", launch_gemm(*qt, x_bf16, m, y, workspace, dev_status,
+                                        static_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

@@ -1,0 +1,41 @@
+// sss_internal.cuh -- declarations shared by the CUDA translation units of
+// the library (not installed; the public interface is include/sss.h).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "sss.h"
+
+namespace sss {
+
+// Number of SMs of the current device (queried once per device).
+int device_sm_count();
+
+// Launchers.  Arguments are validated by the C ABI before these run.
+cudaError_t launch_quantize(const float* w, const sss_qtensor_t& t,
+                            uint8_t* clip_counts, uint32_t* status,
+                            cudaStream_t stream);
+cudaError_t launch_dequantize(const sss_qtensor_t& t, void* out, int out_dtype,
+                              cudaStream_t stream);
+
+size_t gemv_workspace_bytes(const sss_qtensor_t& t, int batch);
+cudaError_t launch_gemv(const sss_qtensor_t& t, const uint16_t* x, int batch,
+                        float* y, void* workspace, cudaStream_t stream);
+
+size_t gemm_workspace_bytes(const sss_qtensor_t& t, int64_t m);
+cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m,
+                        float* y, void* workspace, uint32_t* status,
+                        cudaStream_t stream);
+
+// ---------------------------------------------------------------------------
+// Device helpers
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ bool is_nonfinite(float v) {
+  return (__float_as_uint(v) & 0x7f800000u) == 0x7f800000u;
+}
+
+}  // namespace sss

@@ -1,0 +1,225 @@
+"""Thin ctypes binding of the C ABI in include/sss.h.
+
+Argument marshalling only: every step of the path runs in libsss.so's CUDA
+kernels.  torch supplies device memory and streams.  There is no fallback:
+if the library cannot be built or loaded, these functions raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from dataclasses import dataclass
+from typing import Optional
+
+from . import _build
+
+GRID_UNSIGNED_SYM = 0
+GRID_SIGNED_SYM = 1
+GRID_ASYM = 2
+GRIDS = {"unsigned": GRID_UNSIGNED_SYM, "signed": GRID_SIGNED_SYM, "asym": GRID_ASYM}
+
+OUT_F32, OUT_F16, OUT_BF16 = 0, 1, 2
+OP_GEMV, OP_GEMM = 0, 1
+
+FLAG_NONFINITE = 0x1
+FLAG_RANGE = 0x2
+FLAG_TIMEOUT = 0x4
+
+SSS_OK = 0
+STATUS_NAMES = {0: "SSS_OK", 1: "SSS_E_ARG", 2: "SSS_E_UNSUPPORTED", 3: "SSS_E_ALIGN",
+                4: "SSS_E_CUDA", 5: "SSS_E_WORKSPACE"}
+
+EXPORTS = ("sss_codes_bytes", "sss_status_string", "sss_last_error", "sss_quantize",
+           "sss_dequantize", "sss_gemv", "sss_gemm", "sss_workspace_bytes")
+
+
+class SssError(RuntimeError):
+    def __init__(self, fn: str, status: int, detail: str = ""):
+        self.status = status
+        super().__init__(f"{fn} -> {STATUS_NAMES.get(status, status)}"
+                         + (f" ({detail})" if detail else ""))
+
+
+class QTensorDesc(ctypes.Structure):
+    """Mirror of sss_qtensor_t."""
+    _fields_ = [
+        ("n", ctypes.c_int64),
+        ("k", ctypes.c_int64),
+        ("q", ctypes.c_int32),
+        ("group", ctypes.c_int32),
+        ("grid", ctypes.c_int32),
+        ("reserved", ctypes.c_int32),
+        ("codes", ctypes.c_void_p),
+        ("scales", ctypes.c_void_p),
+        ("mins", ctypes.c_void_p),
+    ]
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_needed: bool = True):
+    """Load libsss.so (building it with nvcc first if it is missing/stale)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if build_if_needed:
+            _build.build()
+        if not os.path.exists(_build.LIB):
+            raise RuntimeError(f"CUDA library missing: {_build.LIB}")
+        L = ctypes.CDLL(_build.LIB)
+        vp, i32, i64, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
+        P = ctypes.POINTER(QTensorDesc)
+        L.sss_codes_bytes.argtypes = [i64, i64, i32]
+        L.sss_codes_bytes.restype = sz
+        L.sss_status_string.argtypes = [i32]
+        L.sss_status_string.restype = ctypes.c_char_p
+        L.sss_last_error.argtypes = []
+        L.sss_last_error.restype = ctypes.c_char_p
+        L.sss_quantize.argtypes = [vp, P, vp, vp, vp]
+        L.sss_quantize.restype = i32
+        L.sss_dequantize.argtypes = [P, vp, i32, vp]
+        L.sss_dequantize.restype = i32
+        L.sss_gemv.argtypes = [P, vp, i32, vp, vp, sz, vp, vp]
+        L.sss_gemv.restype = i32
+        L.sss_gemm.argtypes = [P, vp, i64, vp, vp, sz, vp, vp]
+        L.sss_gemm.restype = i32
+        L.sss_workspace_bytes.argtypes = [P, i64, i32]
+        L.sss_workspace_bytes.restype = sz
+        _lib = L
+        return L
+
+
+def _ptr(t) -> int:
+    return 0 if t is None else int(t.data_ptr())
+
+
+def _stream(stream) -> int:
+    import torch
+
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return int(stream.cuda_stream)
+
+
+def _check(fn: str, st: int):
+    if st != SSS_OK:
+        L = load(False)
+        raise SssError(fn, st, L.sss_last_error().decode())
+
+
+@dataclass
+class QTensor:
+    """A packed weight tensor: torch device buffers plus its shape metadata."""
+    n: int
+    k: int
+    q: int
+    group: int
+    grid: int
+    codes: "object"   # torch.uint8 [n, k*q/8]
+    scales: "object"  # torch.int16 (fp16 bits) [n, k/group]
+    mins: Optional["object"] = None  # torch.int16 [n, k/group] for ASYM
+
+    def desc(self) -> QTensorDesc:
+        return QTensorDesc(self.n, self.k, self.q, self.group, self.grid, 0,
+                           _ptr(self.codes), _ptr(self.scales), _ptr(self.mins))
+
+    @property
+    def nbytes(self) -> int:
+        b = self.codes.numel() + 2 * self.scales.numel()
+        if self.mins is not None:
+            b += 2 * self.mins.numel()
+        return b
+
+
+def empty_qtensor(n: int, k: int, q: int, group: int, grid: int, device="cuda") -> QTensor:
+    import torch
+
+    codes = torch.empty((n, k * q // 8), dtype=torch.uint8, device=device)
+    scales = torch.empty((n, k // group), dtype=torch.int16, device=device)
+    mins = (torch.empty((n, k // group), dtype=torch.int16, device=device)
+            if grid == GRID_ASYM else None)
+    return QTensor(n, k, q, group, grid, codes, scales, mins)
+
+
+# ---------------------------------------------------------------------------
+# entry points (same names as the C ABI)
+# ---------------------------------------------------------------------------
+
+def sss_codes_bytes(n: int, k: int, q: int) -> int:
+    return int(load().sss_codes_bytes(n, k, q))
+
+
+def sss_workspace_bytes(qt: QTensor, m_or_batch: int, op: int) -> int:
+    d = qt.desc()
+    return int(load().sss_workspace_bytes(ctypes.byref(d), m_or_batch, op))
+
+
+def sss_status_string(status: int) -> str:
+    return load().sss_status_string(status).decode()
+
+
+def sss_quantize(w, q: int, group: int, grid: int, out: Optional[QTensor] = None,
+                 clip_counts=None, dev_status=None, stream=None) -> QTensor:
+    """Quantize fp32 weights w [n, k] (CUDA tensor) into a packed QTensor."""
+    n, k = w.shape
+    if out is None:
+        out = empty_qtensor(n, k, q, group, grid, device=w.device)
+    d = out.desc()
+    st = load().sss_quantize(_ptr(w), ctypes.byref(d), _ptr(clip_counts), _ptr(dev_status),
+                             _stream(stream))
+    _check("sss_quantize", st)
+    return out
+
+
+def sss_dequantize(qt: QTensor, out=None, out_dtype: int = OUT_F32, stream=None):
+    import torch
+
+    if out is None:
+        dt = {OUT_F32: torch.float32, OUT_F16: torch.float16, OUT_BF16: torch.bfloat16}[out_dtype]
+        out = torch.empty((qt.n, qt.k), dtype=dt, device=qt.codes.device)
+    d = qt.desc()
+    st = load().sss_dequantize(ctypes.byref(d), _ptr(out), out_dtype, _stream(stream))
+    _check("sss_dequantize", st)
+    return out
+
+
+def sss_gemv(qt: QTensor, x, y=None, workspace=None, dev_status=None, stream=None):
+    """y [batch, n] fp32 = x [batch, k] (bf16) @ dequant(qt)^T."""
+    import torch
+
+    batch = x.shape[0] if x.dim() == 2 else 1
+    if y is None:
+        y = torch.empty((batch, qt.n), dtype=torch.float32, device=x.device)
+    d = qt.desc()
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    st = load().sss_gemv(ctypes.byref(d), _ptr(x), batch, _ptr(y), _ptr(workspace), ws_bytes,
+                         _ptr(dev_status), _stream(stream))
+    _check("sss_gemv", st)
+    return y
+
+
+def sss_gemm(qt: QTensor, x, y=None, workspace=None, dev_status=None, stream=None):
+    """Y [m, n] fp32 = X [m, k] (bf16) @ dequant(qt)^T on the tensor cores."""
+    import torch
+
+    m = x.shape[0]
+    if y is None:
+        y = torch.empty((m, qt.n), dtype=torch.float32, device=x.device)
+    d = qt.desc()
+    if workspace is None:
+        need = int(load().sss_workspace_bytes(ctypes.byref(d), m, OP_GEMM))
+        if need > 0:
+            workspace = torch.empty(need, dtype=torch.uint8, device=x.device)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    st = load().sss_gemm(ctypes.byref(d), _ptr(x), m, _ptr(y), _ptr(workspace), ws_bytes,
+                         _ptr(dev_status), _stream(stream))
+    _check("sss_gemm", st)
+    return y
