@@ -1,0 +1,501 @@
+"""Benchmark of the signed-symmetric few-bit weight path on GB300.
+
+One step = one pass of the whole hot path over one batch of synthetic input,
+on Llama3-8B-shaped linear layers (q/o 4096x4096, k/v 1024x4096, gate/up
+14336x4096, down 4096x14336), signed absmax grid, group 32:
+
+  quantize  one layer's fresh fp32 weights (218.1M weights) at q = 4, 3, 2;
+  GEMV      a batch-1 decode pass over a resident 32-layer packed stack at
+            each of q = 4, 3, 2 (672 GEMVs, 9.2 GB of packed weights);
+  GEMM      a 512-token prefill over the q=4 layer just quantized.
+
+The headline value is the packed-weight GEMV throughput (algorithmic bytes:
+codes + scales + x + y, per launch) in GB/s over the GEMV phases of the
+timed steps; the quantizer (Gweights/s) and GEMM (TFLOP/s) are reported in
+"phases".  Inputs are larger than L2 (the stack alone is 9.2 GB).  Each phase
+is a CUDA graph; phases are timed with CUDA events on the launching stream.
+
+`--impl reference` times the CPU oracle (the plain C reference the tests
+check against) on the host cores on a bounded sample of the same workload.
+
+Launch:  python bench.py [--gpus N] [--steps K] [--warmup W]
+         torchrun --nproc-per-node N bench.py --gpus N ...   (one replica per GPU)
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+MEASURED_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
+QS = (4, 3, 2)
+GROUP = 32
+GEMM_M = 512
+METRIC = ("packed-weight GEMV GB/s at batch 1 (Llama3-8B-shaped layers, q in {2,3,4}, "
+          "group 32, signed symmetric); quantize Gweights/s and GEMM TFLOP/s in phases")
+
+
+def peaks():
+    try:
+        with open(MEASURED_PEAKS) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), float(
+            p.get("bf16_tflops_sustained", p["bf16_tflops"])), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, 1700.0, "fallback"
+
+
+def dist_info():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def traffic_from_profiles(name: str):
+    """dram bytes per launch recorded in profiles/<name> (line
+    'traffic_bytes_per_launch: <int>'), or None."""
+    path = os.path.join(ROOT, "profiles", name)
+    try:
+        for line in open(path):
+            if line.strip().startswith("traffic_bytes_per_launch:"):
+                v = line.split(":", 1)[1].strip()
+                return None if v in ("", "null", "None") else float(v)
+    except OSError:
+        pass
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ---------------------------------------------------------------------------
+# workload
+# ---------------------------------------------------------------------------
+
+class Workload:
+    def __init__(self, layers: int, seed_base: int = 0):
+        import torch
+
+        from paper_2607_08779_gb300 import inputs, sss
+
+        self.torch, self.sss, self.inputs = torch, sss, inputs
+        self.layers = layers
+        self.shapes = list(inputs.LLAMA3_8B_LAYER.items())
+        dev = "cuda"
+        G = sss.GRID_SIGNED_SYM
+        # resident packed stacks, one per q
+        self.stack = {q: [[sss.empty_qtensor(n, k, q, GROUP, G) for _, (n, k) in self.shapes]
+                          for _ in range(layers)] for q in QS}
+        # fresh fp32 layers for the quantize phase (two, alternating), and
+        # the packed outputs of that phase
+        self.fresh = [[torch.empty((n, k), dtype=torch.float32, device=dev)
+                       for _, (n, k) in self.shapes] for _ in range(2)]
+        self.fresh_q = {q: [sss.empty_qtensor(n, k, q, GROUP, G) for _, (n, k) in self.shapes]
+                        for q in QS}
+        tmp = [torch.empty((n, k), dtype=torch.float32, device=dev) for _, (n, k) in self.shapes]
+        for layer in range(layers):
+            for mi, (name, (n, k)) in enumerate(self.shapes):
+                inputs.student_t_weights_cuda(n, k, inputs.weight_seed(2, layer, mi) + seed_base,
+                                              out=tmp[mi])
+                for q in QS:
+                    sss.sss_quantize(tmp[mi], q, GROUP, G, out=self.stack[q][layer][mi])
+        for f in range(2):
+            for mi, (name, (n, k)) in enumerate(self.shapes):
+                inputs.student_t_weights_cuda(n, k, inputs.weight_seed(3, 100 + f, mi) + seed_base,
+                                              out=self.fresh[f][mi])
+        del tmp
+        # activations and outputs
+        ks = sorted({k for _, (n, k) in self.shapes})
+        self.x = {k: inputs.normal_bf16_cuda((1, k), 7 + k + seed_base) for k in ks}
+        self.X = {k: inputs.normal_bf16_cuda((GEMM_M, k), 11 + k + seed_base) for k in ks}
+        self.y = [torch.empty((1, n), dtype=torch.float32, device=dev) for _, (n, k) in self.shapes]
+        self.Y = [torch.empty((GEMM_M, n), dtype=torch.float32, device=dev)
+                  for _, (n, k) in self.shapes]
+        self.ws = {}
+        for mi, (_, (n, k)) in enumerate(self.shapes):
+            need = sss.sss_workspace_bytes(self.fresh_q[4][mi], GEMM_M, sss.OP_GEMM)
+            if need > (self.ws[k].numel() if k in self.ws else -1):
+                self.ws[k] = torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
+        self.status = torch.zeros(1, dtype=torch.int32, device=dev)
+        torch.cuda.synchronize()
+
+        # algorithmic work per step
+        self.gemv_bytes = 0
+        for q in QS:
+            for _, (n, k) in self.shapes:
+                self.gemv_bytes += n * k * q // 8 + 2 * n * (k // GROUP) + 2 * k + 4 * n
+        self.gemv_bytes *= layers
+        self.gemv_launches = layers * len(self.shapes) * len(QS)
+        self.quant_weights = len(QS) * sum(n * k for _, (n, k) in self.shapes)
+        self.quant_bytes = sum(4 * n * k + n * k * q // 8 + 2 * n * (k // GROUP)
+                               for q in QS for _, (n, k) in self.shapes)
+        self.gemm_flops = 2 * GEMM_M * sum(n * k for _, (n, k) in self.shapes)
+        self.launches_per_step = (len(QS) * len(self.shapes) + self.gemv_launches
+                                  + 2 * len(self.shapes))
+
+    # -- phases (each captured once as a CUDA graph) --
+    def quantize_phase(self, f: int):
+        for q in QS:
+            for mi in range(len(self.shapes)):
+                self.sss.sss_quantize(self.fresh[f][mi], q, GROUP, self.sss.GRID_SIGNED_SYM,
+                                      out=self.fresh_q[q][mi], dev_status=self.status)
+
+    def gemv_phase(self):
+        for q in QS:
+            for layer in range(self.layers):
+                for mi, (_, (n, k)) in enumerate(self.shapes):
+                    self.sss.sss_gemv(self.stack[q][layer][mi], self.x[k], y=self.y[mi])
+
+    def gemm_phase(self):
+        for mi, (_, (n, k)) in enumerate(self.shapes):
+            self.sss.sss_gemm(self.fresh_q[4][mi], self.X[k], y=self.Y[mi], workspace=self.ws[k],
+                              dev_status=self.status)
+
+    def capture(self):
+        torch = self.torch
+        # warm every kernel once outside capture
+        self.quantize_phase(0)
+        self.gemv_phase()
+        self.gemm_phase()
+        torch.cuda.synchronize()
+        self.graphs = {}
+        s = torch.cuda.Stream()
+        for key, fn in (("q0", lambda: self.quantize_phase(0)), ("q1", lambda: self.quantize_phase(1)),
+                        ("v", self.gemv_phase), ("m", self.gemm_phase)):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=s):
+                fn()
+            self.graphs[key] = g
+        torch.cuda.synchronize()
+
+    def step(self, s: int, ev):
+        """Replay one step; ev = 4 events recorded around the phases."""
+        ev[0].record()
+        self.graphs["q%d" % (s % 2)].replay()
+        ev[1].record()
+        self.graphs["v"].replay()
+        ev[2].record()
+        self.graphs["m"].replay()
+        ev[3].record()
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    ws, rank, local = dist_info()
+    if ws > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    from paper_2607_08779_gb300 import sss
+
+    sss.load()
+    hbm, bf16, bf16_sus, peak_kind = peaks()
+    wl = Workload(args.layers, seed_base=rank * 7919)
+    wl.capture()
+
+    def barrier():
+        torch.cuda.synchronize()
+        if ws > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    nphase = 4
+    for s in range(args.warmup):
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(nphase)]
+        wl.step(s, ev)
+    barrier()
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.3)
+    events = []
+    start = torch.cuda.Event(enable_timing=True)
+    stop = torch.cuda.Event(enable_timing=True)
+    barrier()
+    start.record()
+    for s in range(args.steps):
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(nphase)]
+        wl.step(s, ev)
+        events.append(ev)
+    stop.record()
+    barrier()
+    clocks = sampler.stop()
+    total_ms = start.elapsed_time(stop)
+    tq = sum(e[0].elapsed_time(e[1]) for e in events)
+    tv = sum(e[1].elapsed_time(e[2]) for e in events)
+    tm = sum(e[2].elapsed_time(e[3]) for e in events)
+    status = int(wl.status.item())
+
+    # the max over ranks of every time; the value counts all ranks' work
+    t = torch.tensor([total_ms, tq, tv, tm], dtype=torch.float64, device="cuda")
+    if ws > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    total_ms, tq, tv, tm = [float(v) for v in t.cpu()]
+    K = args.steps
+    gemv_gbs = ws * wl.gemv_bytes * K / (tv * 1e-3) / 1e9
+    quant_gws = ws * wl.quant_weights * K / (tq * 1e-3) / 1e9
+    quant_gbs = ws * wl.quant_bytes * K / (tq * 1e-3) / 1e9
+    gemm_tfs = ws * wl.gemm_flops * K / (tm * 1e-3) / 1e12
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = measure_e2e(wl, args, ws, barrier)
+
+    # the dominant kernel by time is the GEMV: roofline against HBM
+    per_gpu_gemv = gemv_gbs / ws
+    roofline = {"bound": "hbm", "kernel": "gemv_kernel (decode GEMV, batch 1)",
+                "achieved": round(per_gpu_gemv, 1), "peak": hbm, "unit": "GB/s",
+                "frac": round(per_gpu_gemv / hbm, 4), "peak_source": peak_kind,
+                "traffic": traffic_from_profiles("gemv_llama3_8b_q4_b1.md"),
+                "algorithmic_bytes_per_launch": wl.gemv_bytes // wl.gemv_launches}
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(wl, seconds=args.cpu_seconds)
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(gemv_gbs, 1), "unit": "GB/s", "n_gpus": ws,
+            "steps": K, "warmup": args.warmup, "ms_per_step": round(total_ms / K, 4),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f16", "data": "synthetic",
+            "config": {"workload": "llama3-8b-shaped layers: 32-layer packed stack decode GEMV "
+                                   "(batch 1) at q=4,3,2 + quantize of one fp32 layer at q=4,3,2 "
+                                   "+ 512-token prefill GEMM at q=4",
+                       "layers": args.layers, "q": list(QS), "group": GROUP,
+                       "grid": "signed_symmetric", "batch": 1, "gemm_m": GEMM_M,
+                       "accumulate": "f32", "parallelism": f"replicas x{ws}",
+                       "l2": "inputs larger than L2 (9.2 GB packed stack read per step)"},
+            "roofline": roofline,
+            "phases": {
+                "gemv": {"gbs": round(gemv_gbs, 1), "ms_per_step": round(tv / K, 4),
+                         "frac_hbm": round(per_gpu_gemv / hbm, 4),
+                         "launches_per_step": wl.gemv_launches},
+                "quantize": {"gweights_per_s": round(quant_gws, 1), "gbs": round(quant_gbs, 1),
+                             "frac_hbm": round(quant_gbs / ws / hbm, 4),
+                             "ms_per_step": round(tq / K, 4)},
+                "gemm": {"tflops": round(gemm_tfs, 1), "m": GEMM_M,
+                         "frac_bf16_sustained": round(gemm_tfs / ws / bf16_sus, 4),
+                         "ms_per_step": round(tm / K, 4)},
+            },
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": wl.launches_per_step * K,
+            "clocks": clocks,
+            "device_status": status,
+        }
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def measure_e2e(wl, args, ws, barrier):
+    """The same step through the public API with HOST buffers: the fresh fp32
+    layer, the decode activations and the prefill activations are copied in
+    from pinned host memory, and the outputs read back, inside the region."""
+    torch = wl.torch
+    host_fresh = [f.cpu().pin_memory() for f in wl.fresh[0]]
+    host_x = {k: v.cpu().pin_memory() for k, v in wl.x.items()}
+    host_X = {k: v.cpu().pin_memory() for k, v in wl.X.items()}
+    host_y = [y.cpu().pin_memory() for y in wl.y]
+    host_Y = [Y.cpu().pin_memory() for Y in wl.Y]
+    h2d = sum(t.numel() * t.element_size() for t in host_fresh)
+    h2d += sum(t.numel() * t.element_size() for t in host_x.values())
+    h2d += sum(t.numel() * t.element_size() for t in host_X.values())
+    d2h = sum(t.numel() * t.element_size() for t in host_y + host_Y)
+    steps = max(1, min(args.steps, 5))
+
+    def one():
+        for d, h in zip(wl.fresh[0], host_fresh):
+            d.copy_(h, non_blocking=True)
+        for k in wl.x:
+            wl.x[k].copy_(host_x[k], non_blocking=True)
+            wl.X[k].copy_(host_X[k], non_blocking=True)
+        wl.graphs["q0"].replay()
+        wl.graphs["v"].replay()
+        wl.graphs["m"].replay()
+        for h, d in zip(host_y, wl.y):
+            h.copy_(d, non_blocking=True)
+        for h, d in zip(host_Y, wl.Y):
+            h.copy_(d, non_blocking=True)
+
+    one()
+    barrier()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(steps):
+        one()
+    b.record()
+    barrier()
+    ms = a.elapsed_time(b) / steps
+    t = torch.tensor([ms], dtype=torch.float64, device="cuda")
+    if ws > 1:
+        import torch.distributed as dist
+
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms = float(t.item())
+    return {"value": round(ws * wl.gemv_bytes / (ms * 1e-3) / 1e9, 1), "unit": "GB/s",
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "ms_per_step": round(ms, 4), "steps": steps}
+
+
+def oracle_gemv_rate(codes, scales, n_rows, k, q, xbits, seconds):
+    """GB/s of packed bytes the oracle GEMV processes on this host (one
+    core), over as many row blocks as fit in `seconds`."""
+    import oracle
+
+    rows_per_call = 64
+    row_bytes = k * q // 8 + 2 * (k // GROUP)
+    done_rows, t0 = 0, time.perf_counter()
+    r0 = 0
+    while time.perf_counter() - t0 < seconds:
+        r1 = min(n_rows, r0 + rows_per_call)
+        oracle.gemv(codes[r0:r1], scales[r0:r1], None, r1 - r0, k, q, GROUP,
+                    oracle.GRID_SIGNED_SYM, xbits)
+        done_rows += r1 - r0
+        r0 = 0 if r1 >= n_rows else r1
+    el = time.perf_counter() - t0
+    return done_rows * row_bytes / el / 1e9, done_rows, el
+
+
+def cpu_baseline(wl, seconds: float):
+    """The oracle's GEMV, as it stands, on the host cores, on a bounded
+    sample of the same workload (rows of the layer-0 gate_proj at q=4)."""
+    mi = [name for name, _ in wl.shapes].index("gate_proj")
+    qt = wl.stack[4][0][mi]
+    n, k = qt.n, qt.k
+    codes = qt.codes[:4096].cpu().numpy()
+    scales = qt.scales[:4096].cpu().numpy().view(np.uint16)
+    xbits = wl.x[k].cpu().view(wl.torch.int16).numpy().view(np.uint16)
+    gbs, rows, el = oracle_gemv_rate(codes, scales, codes.shape[0], k, 4, xbits, seconds)
+    return {"value": round(gbs, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": f"{rows} rows of gate_proj (14336x4096) at q=4 g=32, batch 1, "
+                      f"{el:.1f} s of single-threaded oracle GEMV (fp64)"}
+
+
+def run_reference(args):
+    """The oracle on the host cores, on the same metric; rank 0 only."""
+    ws, rank, local = dist_info()
+    if rank != 0:
+        return
+    import oracle
+    from paper_2607_08779_gb300 import inputs
+
+    oracle.build()
+    n, k = inputs.LLAMA3_8B_LAYER["gate_proj"]
+    rows = 1024
+    W = inputs.student_t_weights(rows, k, inputs.weight_seed(2, 0, 4))
+    packed = {}
+    for q in QS:
+        codes, scales, _, _, _ = oracle.quantize(W, q, GROUP, oracle.GRID_SIGNED_SYM)
+        packed[q] = (codes, scales)
+    xbits = inputs.normal_bf16_bits((1, k), 7)
+    per_step = max(0.5, args.ref_seconds)
+    for _ in range(args.warmup):
+        oracle_gemv_rate(*packed[4], rows, k, 4, xbits, 0.05)
+    total_bytes, total_s, t_all = 0.0, 0.0, time.perf_counter()
+    for s in range(args.steps):
+        q = QS[s % len(QS)]
+        gbs, r, el = oracle_gemv_rate(*packed[q], rows, k, q, xbits, per_step)
+        total_bytes += gbs * el * 1e9
+        total_s += el
+    value = total_bytes / total_s / 1e9
+    line = {
+        "metric": METRIC, "value": round(value, 4), "unit": "GB/s", "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(total_s / args.steps * 1e3, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "impl": "reference",
+        "config": {"workload": "llama3-8b-shaped layers: batch-1 GEMV over packed gate_proj "
+                               "rows at q=4,3,2 (bounded sample per step)",
+                   "group": GROUP, "grid": "signed_symmetric", "batch": 1},
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+                         "sample": f"{args.steps} steps x {per_step:.1f} s of oracle GEMV over "
+                                   f"{rows} rows of gate_proj, q cycling 4,3,2"},
+        "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--layers", type=int, default=32)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--ref-seconds", type=float, default=2.0)
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

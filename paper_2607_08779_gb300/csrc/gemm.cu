@@ -496,8 +496,7 @@ cudaError_t run_gemm(const sss_qtensor_t& t, const __half* x16, int64_t m, float
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
   auto kern = gemm_kernel<Q, ASYM, BN, STAGES>;
-  cudaError_t e =
-      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::TOTAL);
+  cudaError_t e = ensure_smem(kern, S::TOTAL);
   if (e != cudaSuccess) return e;
   GemmArgs a;
   a.codes = t.codes;

@@ -449,8 +449,7 @@ template <int Q, bool ASYM, int NB, int RT>
 cudaError_t run(const sss_qtensor_t& t, const uint16_t* x, int batch, float* y,
                 const Plan& p, cudaStream_t stream) {
   auto kern = gemv_kernel<Q, ASYM, NB, RT>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(p.smem));
+  cudaError_t e = ensure_smem(kern, static_cast<int>(p.smem));
   if (e != cudaSuccess) return e;
   GemvArgs a;
   a.codes = t.codes;

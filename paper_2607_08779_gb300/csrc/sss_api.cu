@@ -1,7 +1,9 @@
 // sss_api.cu -- the C ABI declared in include/sss.h: synchronous argument
 // validation, dispatch to the kernels' launchers, and error mapping.  No
 // entry point allocates device memory.
+#include <map>
 #include <mutex>
+#include <utility>
 #include <stdio.h>
 #include <string.h>
 
@@ -47,6 +49,20 @@ sss_status_t finish(const char* what, cudaError_t e) {
 }
 
 }  // namespace
+
+cudaError_t ensure_smem_impl(const void* kernel, int bytes) {
+  static std::mutex mu;
+  static std::map<std::pair<const void*, int>, int> configured;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  int& have = configured[std::make_pair(kernel, dev)];
+  if (have >= bytes) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) have = bytes;
+  return e;
+}
 
 int device_sm_count() {
   static std::mutex mu;

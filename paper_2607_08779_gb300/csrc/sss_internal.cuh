@@ -30,6 +30,15 @@ cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m,
                         float* y, void* workspace, uint32_t* status,
                         cudaStream_t stream);
 
+// Raise a kernel's dynamic shared-memory limit once per (kernel, device)
+// (the call is not stream-ordered; doing it once keeps launches cheap and
+// capturable in CUDA graphs).
+cudaError_t ensure_smem_impl(const void* kernel, int bytes);
+template <typename K>
+cudaError_t ensure_smem(K kernel, int bytes) {
+  return ensure_smem_impl(reinterpret_cast<const void*>(kernel), bytes);
+}
+
 // ---------------------------------------------------------------------------
 // Device helpers
 // ---------------------------------------------------------------------------
