@@ -6,7 +6,9 @@ on Llama3-8B-shaped linear layers (q/o 4096x4096, k/v 1024x4096, gate/up
 
   quantize  one layer's fresh fp32 weights (218.1M weights) at q = 4, 3, 2;
   GEMV      a batch-1 decode pass over a resident 32-layer packed stack at
-            each of q = 4, 3, 2 (672 GEMVs, 9.2 GB of packed weights);
+            each of q = 4, 3, 2 (224 matrices, 9.2 GB of packed weights),
+            launched per layer as a decoder can: {q,k,v} fused, o, {gate,up}
+            fused, down (384 launches, programmatic dependent launch);
   GEMM      a 512-token prefill over the q=4 layer just quantized.
 
 The headline value is the packed-weight GEMV throughput (algorithmic bytes:
@@ -180,13 +182,19 @@ class Workload:
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
         torch.cuda.synchronize()
 
-        # algorithmic work per step
+        # algorithmic work per step: per launch, the codes and scales of its
+        # matrices, its activation vector once, and its outputs
+        dims = dict(self.shapes)
         self.gemv_bytes = 0
         for q in QS:
-            for _, (n, k) in self.shapes:
-                self.gemv_bytes += n * k * q // 8 + 2 * n * (k // GROUP) + 2 * k + 4 * n
+            for grp in self.GROUPS:
+                k = dims[grp[0]][1]
+                self.gemv_bytes += 2 * k
+                for nm in grp:
+                    n = dims[nm][0]
+                    self.gemv_bytes += n * k * q // 8 + 2 * n * (k // GROUP) + 4 * n
         self.gemv_bytes *= layers
-        self.gemv_launches = layers * len(self.shapes) * len(QS)
+        self.gemv_launches = layers * len(self.GROUPS) * len(QS)
         self.quant_weights = len(QS) * sum(n * k for _, (n, k) in self.shapes)
         self.quant_bytes = sum(4 * n * k + n * k * q // 8 + 2 * n * (k // GROUP)
                                for q in QS for _, (n, k) in self.shapes)
@@ -201,11 +209,24 @@ class Workload:
                 self.sss.sss_quantize(self.fresh[f][mi], q, GROUP, self.sss.GRID_SIGNED_SYM,
                                       out=self.fresh_q[q][mi], dev_status=self.status)
 
+    # one decode token through a layer: the launches a decoder can issue, in
+    # its dependency order -- {q, k, v} share x, then o, then {gate, up}
+    # share x, then down -- each a programmatic dependent launch (the
+    # resident weights are not written by the preceding kernels)
+    GROUPS = (("q_proj", "k_proj", "v_proj"), ("o_proj",), ("gate_proj", "up_proj"),
+              ("down_proj",))
+
     def gemv_phase(self):
+        sss = self.sss
+        idx = {name: i for i, (name, _) in enumerate(self.shapes)}
+        flags = sss.GEMV_PDL | sss.GEMV_WEIGHTS_READY
         for q in QS:
             for layer in range(self.layers):
-                for mi, (_, (n, k)) in enumerate(self.shapes):
-                    self.sss.sss_gemv(self.stack[q][layer][mi], self.x[k], y=self.y[mi])
+                for grp in self.GROUPS:
+                    mis = [idx[nm] for nm in grp]
+                    k = self.shapes[mis[0]][1][1]
+                    sss.sss_gemv_multi([self.stack[q][layer][mi] for mi in mis], self.x[k][0],
+                                       ys=[self.y[mi][0] for mi in mis], flags=flags)
 
     def gemm_phase(self):
         for mi, (_, (n, k)) in enumerate(self.shapes):
@@ -323,6 +344,8 @@ def run_ours(args):
                                    "+ 512-token prefill GEMM at q=4",
                        "layers": args.layers, "q": list(QS), "group": GROUP,
                        "grid": "signed_symmetric", "batch": 1, "gemm_m": GEMM_M,
+                       "decode_launches_per_layer": "{q,k,v} fused, o, {gate,up} fused, down; "
+                                                    "programmatic dependent launch",
                        "accumulate": "f32", "parallelism": f"replicas x{ws}",
                        "l2": "inputs larger than L2 (9.2 GB packed stack read per step)"},
             "roofline": roofline,
@@ -479,6 +502,90 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def run_micro(args):
+    """One operation on one Llama3-8B shape, cycling over `--rotate` distinct
+    copies of its inputs (more than L2 in total), timed with CUDA events.
+    Prints one JSON line (not the benchmark's headline line)."""
+    import torch
+
+    from paper_2607_08779_gb300 import inputs, sss
+
+    torch.cuda.set_device(0)
+    sss.load()
+    names = args.matrices.split(",")
+    shapes = [inputs.LLAMA3_8B_LAYER[nm] for nm in names]
+    k = shapes[0][1]
+    G = sss.GRID_ASYM if args.grid == "asym" else (
+        sss.GRID_UNSIGNED_SYM if args.grid == "unsigned" else sss.GRID_SIGNED_SYM)
+    q, g = args.q, args.group
+    copies = []
+    for c in range(args.rotate):
+        mats = []
+        for mi, (n, kk) in enumerate(shapes):
+            w = inputs.student_t_weights_cuda(n, kk, 1000 * c + mi)
+            if args.micro == "quantize":
+                mats.append((w, sss.empty_qtensor(n, kk, q, g, G)))
+            else:
+                mats.append(sss.sss_quantize(w, q, g, G))
+                del w
+        copies.append(mats)
+    x = inputs.normal_bf16_cuda((args.m if args.micro == "gemm" else 1, k), 5)
+    ys = [torch.empty((args.m if args.micro == "gemm" else 1, n), dtype=torch.float32,
+                      device="cuda") for n, _ in shapes]
+    ws = None
+    if args.micro == "gemm":
+        ws = torch.empty(max(sss.sss_workspace_bytes(copies[0][0], args.m, sss.OP_GEMM), 16),
+                         dtype=torch.uint8, device="cuda")
+
+    def op(c):
+        mats = copies[c % args.rotate]
+        if args.micro == "gemv":
+            sss.sss_gemv_multi(mats, x[0], ys=[y[0] for y in ys], flags=args.flags)
+        elif args.micro == "gemv_single":
+            for qt, y in zip(mats, ys):
+                sss.sss_gemv(qt, x, y=y)
+        elif args.micro == "gemm":
+            for qt, y in zip(mats, ys):
+                sss.sss_gemm(qt, x, y=y, workspace=ws)
+        else:
+            for w, qt in mats:
+                sss.sss_quantize(w, q, g, G, out=qt)
+
+    for c in range(3):
+        op(c)
+    torch.cuda.synchronize()
+    # the timed loop is one CUDA graph, so host-side call overhead is excluded
+    graph = torch.cuda.CUDAGraph()
+    cs = torch.cuda.Stream()
+    with torch.cuda.graph(graph, stream=cs):
+        for c in range(args.iters):
+            op(c)
+    graph.replay()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    graph.replay()
+    b.record()
+    torch.cuda.synchronize()
+    us = a.elapsed_time(b) * 1e3 / args.iters
+    nbytes = 0
+    for (n, kk) in shapes:
+        packed = n * kk * q // 8 + 2 * n * (kk // g) * (2 if G == sss.GRID_ASYM else 1)
+        if args.micro == "quantize":
+            nbytes += 4 * n * kk + packed
+        elif args.micro == "gemm":
+            nbytes += packed + 2 * args.m * kk + 4 * args.m * n
+        else:
+            nbytes += packed + 4 * n
+    if args.micro != "quantize":
+        nbytes += 2 * k * (args.m if args.micro == "gemm" else 1)
+    flops = 2 * (args.m if args.micro == "gemm" else 1) * sum(n * kk for n, kk in shapes)
+    print(json.dumps({"micro": args.micro, "matrices": names, "q": q, "group": g,
+                      "grid": args.grid, "us_per_call": round(us, 3),
+                      "gbs": round(nbytes / us / 1e3, 1), "tflops": round(flops / us / 1e6, 2),
+                      "iters": args.iters, "rotate": args.rotate}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -490,7 +597,19 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--ref-seconds", type=float, default=2.0)
+    ap.add_argument("--micro", choices=["gemv", "gemv_single", "gemm", "quantize"])
+    ap.add_argument("--matrices", default="gate_proj,up_proj")
+    ap.add_argument("--q", type=int, default=4)
+    ap.add_argument("--group", type=int, default=32)
+    ap.add_argument("--grid", choices=["signed", "unsigned", "asym"], default="signed")
+    ap.add_argument("--m", type=int, default=512)
+    ap.add_argument("--iters", type=int, default=50)
+    ap.add_argument("--rotate", type=int, default=8)
+    ap.add_argument("--flags", type=int, default=0)
     args = ap.parse_args()
+    if args.micro:
+        run_micro(args)
+        return
     if args.impl == "reference":
         run_reference(args)
     else:

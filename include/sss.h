@@ -109,14 +109,15 @@ const char* sss_last_error(void);
  *
  *   w           [in]  device fp32 [n][k], 16-byte aligned, row-major contiguous.
  *   out         [in]  descriptor of the outputs (n, k, q, group, grid and the
- *                     device buffers codes, scales, mins); not retained.
+ *                     device buffers codes (16-byte aligned), scales, mins);
+ *                     not retained.
  *   clip_counts [out] nullable device uint8 [n][k/group][2]: for symmetric
  *                     grids {|C_gamma|, |C_-gamma|} (def:clipped-set): the
  *                     number of pre-clip codes equal to +2^(q-1) and to
  *                     -2^(q-1); for ASYM {0, 0}.
  *   dev_status  [out] nullable device uint32; SSS_FLAG_NONFINITE/RANGE OR-ed.
  * Errors: SSS_E_ARG (q, group, grid, k % group, NULL buffers), SSS_E_ALIGN
- * (w not 16-byte aligned), SSS_E_CUDA.  n == 0 is a no-op.
+ * (w or codes not 16-byte aligned), SSS_E_CUDA.  n == 0 is a no-op.
  */
 sss_status_t sss_quantize(const float* w, const sss_qtensor_t* out,
                           uint8_t* clip_counts, uint32_t* dev_status,
@@ -153,6 +154,35 @@ sss_status_t sss_dequantize(const sss_qtensor_t* qt, void* out,
 sss_status_t sss_gemv(const sss_qtensor_t* qt, const uint16_t* x_bf16,
                       int32_t batch, float* y, void* workspace,
                       size_t ws_bytes, uint32_t* dev_status, void* stream);
+
+/* flags of sss_gemv_multi */
+#define SSS_GEMV_PDL 0x1u           /* launch as a programmatic dependent launch: the kernel
+                                       may start while the preceding kernel in the stream
+                                       drains; it reads x (and writes y) only after that
+                                       kernel has completed                                */
+#define SSS_GEMV_WEIGHTS_READY 0x2u /* with SSS_GEMV_PDL: the packed weights are not written
+                                       by the preceding work in the stream, so they may be
+                                       streamed in before it completes                     */
+
+/*
+ * sss_gemv_multi -- batch-1 decode GEMV of several packed matrices that
+ * share one activation vector (e.g. the q/k/v or gate/up projections of a
+ * layer) in one launch: y_j[r] = sum_k w^_j[r][k] * x[k] (same arithmetic as
+ * sss_gemv).  The weights are streamed through shared memory by bulk copies.
+ *   qts     [in]  count pointers to packed tensors with equal k, q, group and
+ *                 grid; codes, scales (and mins) 16-byte aligned.
+ *   ys      [out] count device fp32 pointers, y_j of length qts[j]->n.
+ *   count   [in]  1..4.
+ *   x_bf16  [in]  device bf16 [k], 16-byte aligned.
+ *   flags   [in]  SSS_GEMV_* bits.
+ *   dev_status [out] nullable; SSS_FLAG_TIMEOUT if a bounded wait expired.
+ * Shapes with k % 256 != 0 or k % (8*group) != 0, or unaligned buffers, run
+ * as one sss_gemv per matrix (flags then have no effect).
+ * Errors: SSS_E_ARG, SSS_E_ALIGN, SSS_E_CUDA.
+ */
+sss_status_t sss_gemv_multi(const sss_qtensor_t* const* qts, float* const* ys,
+                            int32_t count, const uint16_t* x_bf16, uint32_t flags,
+                            uint32_t* dev_status, void* stream);
 
 /*
  * sss_gemm -- prefill GEMM Y[m][r] = sum_k w^[r][k] * X[m][k] (Appendix B.3,

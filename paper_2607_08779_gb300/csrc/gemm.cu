@@ -346,55 +346,76 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int64_t nG = a.k / a.G;
     const uint8_t* rowp = a.codes + (rok ? r : 0) * (a.k * Q / 8);
     const int sw = i & 7;  // swizzle phase of this row
-    bool ok = true;
-    for (int kb = 0; kb < nkb && ok; ++kb) {
-      const int s = kb % STAGES;
-      const uint32_t ph = static_cast<uint32_t>(kb / STAGES) & 1u;
-      if (!mbar_wait(&empty[s], ph ^ 1u, abort)) {
-        ok = false;
-        break;
-      }
-      unsigned char* arow = smem + s * S::STAGE + (i >> 3) * 1024 + sw * 128;
+    // codes and scales of one 64-wide k-block of this row
+    struct KBlock {
+      uint32_t w[2][4];
+      uint16_t s[2], m[2];
+    };
+    auto fetch = [&](KBlock& d, int kb) {
+      if (kb >= nkb) return;
 #pragma unroll
-      for (int j = 0; j < 2; ++j) {  // two 32-code sub-chunks per 64-wide k-block
+      for (int j = 0; j < 2; ++j) {
         const int64_t kc = static_cast<int64_t>(kb) * kBK + 32 * j;
         const int64_t grp = kc / a.G;
         const int sc = static_cast<int>((kc % a.G) / 32);
-        uint32_t w[4];
-        load_sub32<Q>(rowp, grp, sc, a.G, rok, w);
-        __half2 s2 = __float2half2_rn(0.f), m2 = __float2half2_rn(0.f);
-        if (rok) {
-          const __half sh = __ushort_as_half(a.scales[r * nG + grp]);
-          s2 = __halves2half2(sh, sh);
+        load_sub32<Q>(rowp, grp, sc, a.G, rok, d.w[j]);
+        d.s[j] = rok ? __ldcs(a.scales + r * nG + grp) : static_cast<uint16_t>(0);
+        if constexpr (ASYM) d.m[j] = rok ? __ldcs(a.mins + r * nG + grp) : static_cast<uint16_t>(0);
+      }
+    };
+    // the global loads run kPrefetch k-blocks ahead of their use
+    constexpr int kPrefetch = 4;
+    KBlock ring[kPrefetch];
+#pragma unroll
+    for (int q0 = 0; q0 < kPrefetch; ++q0) fetch(ring[q0], q0);
+    bool ok = true;
+    for (int kb0 = 0; kb0 < nkb && ok; kb0 += kPrefetch) {
+#pragma unroll
+      for (int q0 = 0; q0 < kPrefetch; ++q0) {
+        const int kb = kb0 + q0;
+        if (kb >= nkb || !ok) break;
+        const int s = kb % STAGES;
+        const uint32_t ph = static_cast<uint32_t>(kb / STAGES) & 1u;
+        if (!mbar_wait(&empty[s], ph ^ 1u, abort)) {
+          ok = false;
+          break;
+        }
+        unsigned char* arow = smem + s * S::STAGE + (i >> 3) * 1024 + sw * 128;
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {  // two 32-code sub-chunks per 64-wide k-block
+          const __half sh = __ushort_as_half(ring[q0].s[j]);
+          const __half2 s2 = __halves2half2(sh, sh);
+          __half2 m2 = __float2half2_rn(0.f);
           if constexpr (ASYM) {
-            const __half mh = __ushort_as_half(a.mins[r * nG + grp]);
+            const __half mh = __ushort_as_half(ring[q0].m[j]);
             m2 = __halves2half2(mh, mh);
           }
-        }
-        uint32_t u[16];
-        code_pairs<Q>(w, u);
-        uint32_t out[16];
+          uint32_t u[16];
+          code_pairs<Q>(ring[q0].w[j], u);
+          uint32_t out[16];
 #pragma unroll
-        for (int p = 0; p < 16; ++p) {
-          // 1024 + u as fp16, minus 1024 (+ 2^(q-1) for symmetric codes): exact
-          const uint32_t mag = u[p] | 0x64006400u;
-          __half2 hv = *reinterpret_cast<const __half2*>(&mag);
-          const __half2 bias = ASYM ? __float2half2_rn(1024.f)
-                                    : __float2half2_rn(static_cast<float>(1024 + (1 << (Q - 1))));
-          hv = __hsub2(hv, bias);                                  // c (or u) exactly
-          hv = ASYM ? __hfma2(hv, s2, m2) : __hmul2(hv, s2);       // RN16(s*c) / RN16(s*u+m)
-          out[p] = *reinterpret_cast<const uint32_t*>(&hv);
-        }
+          for (int p = 0; p < 16; ++p) {
+            // 1024 + u as fp16, minus 1024 (+ 2^(q-1) for symmetric codes): exact
+            const uint32_t mag = u[p] | 0x64006400u;
+            __half2 hv = *reinterpret_cast<const __half2*>(&mag);
+            const __half2 bias = ASYM ? __float2half2_rn(1024.f)
+                                      : __float2half2_rn(static_cast<float>(1024 + (1 << (Q - 1))));
+            hv = __hsub2(hv, bias);                               // c (or u) exactly
+            hv = ASYM ? __hfma2(hv, s2, m2) : __hmul2(hv, s2);    // RN16(s*c) / RN16(s*u+m)
+            out[p] = *reinterpret_cast<const uint32_t*>(&hv);
+          }
 #pragma unroll
-        for (int cc = 0; cc < 4; ++cc) {  // four 16-byte chunks of 8 elements
-          const int chunk = 4 * j + cc;
-          uint4 v = make_uint4(out[4 * cc], out[4 * cc + 1], out[4 * cc + 2], out[4 * cc + 3]);
-          *reinterpret_cast<uint4*>(arow + ((chunk ^ sw) << 4)) = v;
+          for (int cc = 0; cc < 4; ++cc) {  // four 16-byte chunks of 8 elements
+            const int chunk = 4 * j + cc;
+            uint4 v = make_uint4(out[4 * cc], out[4 * cc + 1], out[4 * cc + 2], out[4 * cc + 3]);
+            *reinterpret_cast<uint4*>(arow + ((chunk ^ sw) << 4)) = v;
+          }
         }
+        fence_proxy_async_smem();  // generic-proxy stores -> visible to the tensor core
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&full_a[s]);
+        fetch(ring[q0], kb + kPrefetch);
       }
-      fence_proxy_async_smem();  // generic-proxy stores -> visible to the tensor core
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&full_a[s]);
     }
     // ---------------- epilogue ----------------
     if (ok && mbar_wait(done, 0, abort)) {
@@ -455,25 +476,6 @@ __global__ void __launch_bounds__(256)
 // host side
 // ---------------------------------------------------------------------------
 
-using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
-                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
-                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
-                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFn encode_fn() {
-  static std::once_flag once;
-  static EncodeTiledFn fn = nullptr;
-  std::call_once(once, [] {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<EncodeTiledFn>(p);
-  });
-  return fn;
-}
-
 size_t x16_bytes(int64_t m, int64_t k) {
   return (static_cast<size_t>(m) * static_cast<size_t>(k) * 2 + 255) / 256 * 256;
 }
@@ -483,7 +485,7 @@ cudaError_t run_gemm(const sss_qtensor_t& t, const __half* x16, int64_t m, float
                      uint32_t* status, cudaStream_t stream) {
   constexpr int STAGES = (BN == 256) ? 4 : 6;
   using S = Smem<BN, STAGES>;
-  EncodeTiledFn enc = encode_fn();
+  EncodeTiledFn enc = tensor_map_encoder();
   if (enc == nullptr) return cudaErrorNotSupported;
   CUtensorMap map;
   const cuuint64_t dims[2] = {static_cast<cuuint64_t>(t.k), static_cast<cuuint64_t>(m)};

@@ -47,7 +47,6 @@ namespace {
 
 constexpr int kMaxWarps = 4;
 constexpr int kMaxKS = 8;
-constexpr int kWindowGroups = 128;  // groups of x staged per CTA at once (batch 1)
 
 template <int Q>
 struct QT;
@@ -175,6 +174,16 @@ __host__ __device__ __forceinline__ int pitch_bytes(int q, int G) {
   return (G / 32) * (q == 3 ? 128 : 64) + 16;
 }
 
+// Registers of one work unit: the codes of one 32-code sub-chunk (sc) of the
+// lane's two groups (h = 0, 1) for its RT x 2 rows, plus, for the first
+// sub-chunk of a step, the fp16 scales (and mins) of those groups.
+template <int Q, int RT>
+struct Unit {
+  uint32_t w[2][RT][2][QT<Q>::NW];
+  uint32_t s[RT][2];  // two fp16: groups 2t and 2t+1 of the step
+  uint32_t m[RT][2];
+};
+
 template <int Q, bool ASYM, int NB, int RT>
 __global__ void __launch_bounds__(kMaxWarps * 32)
     gemv_kernel(const GemvArgs a) {
@@ -184,13 +193,13 @@ __global__ void __launch_bounds__(kMaxWarps * 32)
   extern __shared__ __align__(16) unsigned char smem[];
 
   const int G = a.G;
-  const int SC = G / 32;                     // sub-chunks per group
+  const int SC = G / 32;  // 32-code sub-chunks per group
   const int pitch = pitch_bytes(Q, G);
   const int wg = a.window_groups;
   const int nwarps = blockDim.x >> 5;
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int gq = lane >> 2, tq = lane & 3;   // mma fragment coordinates
+  const int gq = lane >> 2, tq = lane & 3;  // mma fragment coordinates
   const int64_t nG = a.k / G;
 
   // shared memory: [NB][wg][pitch] arranged activations | zero block |
@@ -206,10 +215,11 @@ __global__ void __launch_bounds__(kMaxWarps * 32)
   const int64_t nsteps_total = (nG + 7) / 8;
   const int64_t step_hi = min(step_lo + a.steps_per_cta, nsteps_total);
   const int64_t row_bytes = a.k * Q / 8;
-  const int64_t gpr = nG;  // groups per row (scale row stride)
 
   // rows this lane feeds: tile tt, half hh -> row0 + 16*tt + gq + 8*hh
   const uint8_t* rowp[RT][2];
+  const uint16_t* srow[RT][2];
+  const uint16_t* mrow[RT][2];
   bool rowok[RT][2];
 #pragma unroll
   for (int tt = 0; tt < RT; ++tt)
@@ -217,155 +227,202 @@ __global__ void __launch_bounds__(kMaxWarps * 32)
     for (int hh = 0; hh < 2; ++hh) {
       const int64_t r = row0 + 16 * tt + gq + 8 * hh;
       rowok[tt][hh] = r < a.n;
-      rowp[tt][hh] = a.codes + (rowok[tt][hh] ? r : 0) * row_bytes;
+      const int64_t rr = rowok[tt][hh] ? r : 0;
+      rowp[tt][hh] = a.codes + rr * row_bytes;
+      srow[tt][hh] = a.scales + rr * nG;
+      mrow[tt][hh] = ASYM ? a.mins + rr * nG : nullptr;
     }
+
+  // unit u of this warp in the window starting at step wstep:
+  // step = wstep + warp + (u / SC) * nwarps, sc = u % SC
+  auto load_unit = [&](Unit<Q, RT>& U, int64_t step, int sc) {
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int64_t grp = step * 8 + 2 * tq + h;
+      const bool gok = grp < nG;
+#pragma unroll
+      for (int tt = 0; tt < RT; ++tt)
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh)
+          load_sub<Q>(rowp[tt][hh], static_cast<int>(grp), sc, G, gok && rowok[tt][hh],
+                      U.w[h][tt][hh]);
+    }
+    if (sc == 0) {
+      const int64_t g0 = step * 8 + 2 * tq;
+#pragma unroll
+      for (int tt = 0; tt < RT; ++tt)
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+          uint32_t lo = 0, hi = 0, mlo = 0, mhi = 0;
+          if (rowok[tt][hh] && g0 < nG) {
+            lo = __ldcs(srow[tt][hh] + g0);
+            if constexpr (ASYM) mlo = __ldcs(mrow[tt][hh] + g0);
+          }
+          if (rowok[tt][hh] && g0 + 1 < nG) {
+            hi = __ldcs(srow[tt][hh] + g0 + 1);
+            if constexpr (ASYM) mhi = __ldcs(mrow[tt][hh] + g0 + 1);
+          }
+          U.s[tt][hh] = lo | (hi << 16);
+          U.m[tt][hh] = mlo | (mhi << 16);
+        }
+    }
+  };
 
   float acc[NB][RT][2];
 #pragma unroll
   for (int b = 0; b < NB; ++b)
 #pragma unroll
     for (int tt = 0; tt < RT; ++tt) acc[b][tt][0] = acc[b][tt][1] = 0.f;
+  float d[NB][RT][4];
+  uint32_t st[RT][2], mt[RT][2];  // scales of the step being accumulated
 
   for (int i = threadIdx.x; i < 32; i += blockDim.x) reinterpret_cast<uint32_t*>(zero)[i] = 0u;
 
+  Unit<Q, RT> ua, ub;
   for (int64_t wstep = step_lo; wstep < step_hi; wstep += wg / 8) {
     const int64_t wgrp0 = wstep * 8;  // first group of the window
     const int64_t wsteps_end = min(step_hi, wstep + wg / 8);
     const int ngrp_win = static_cast<int>(min(static_cast<int64_t>(wg), nG - wgrp0));
+    const int64_t my_steps =
+        (wstep + warp < wsteps_end) ? (wsteps_end - (wstep + warp) + nwarps - 1) / nwarps : 0;
+    const int nunits = static_cast<int>(my_steps) * SC;
 
-    // ---- stage the window's activations in mma order, and group sums ----
-    __syncthreads();
-    {
-      const int per_group = SC * NP;  // pairs per group
-      const int total = NB * ngrp_win * per_group;
-      for (int i = threadIdx.x; i < total; i += blockDim.x) {
-        const int b = i / (ngrp_win * per_group);
-        const int rem = i - b * ngrp_win * per_group;
-        const int gl = rem / per_group;
-        const int pi = rem - gl * per_group;
-        const int sc = pi / NP, p = pi - sc * NP;
-        int ea, eb;
-        float mult;
-        pair_desc<Q>(p, ea, eb, mult);
-        __half2 hv = __floats2half2_rn(0.f, 0.f);
+    // the first unit's code loads go out before the activations are staged
+    if (nunits > 0) load_unit(ua, wstep + warp, 0);
+
+    __syncthreads();  // previous window fully consumed
+    // ---- stage activations in mma order (one thread per batch row x group) ----
+    for (int it = threadIdx.x; it < NB * ngrp_win; it += blockDim.x) {
+      const int b = it / ngrp_win, gl = it - b * ngrp_win;
+      unsigned char* dst = xs + (static_cast<size_t>(b) * wg + gl) * pitch;
+      float sum = 0.f;
+      for (int sc = 0; sc < SC; ++sc) {
+        float xv[32];
         if (b < a.batch) {
-          const uint16_t* xr = a.x + static_cast<int64_t>(b) * a.k +
-                               (wgrp0 + gl) * G + sc * 32;
-          const float xa = __bfloat162float(__ushort_as_bfloat16(xr[ea]));
-          const float xb = __bfloat162float(__ushort_as_bfloat16(xr[eb]));
-          hv = __floats2half2_rn(xa * mult, xb * mult);
-        }
-        *reinterpret_cast<__half2*>(xs + (static_cast<size_t>(b) * wg + gl) * pitch +
-                                    sc * NP * 4 + p * 4) = hv;
-      }
-      // bias terms: symmetric  -2^(q-1) * 2^-24 * sum_{k in g} x
-      //             asymmetric  2^-24 * sum_{k in g} x  (multiplied by m later)
-      const int nbias = NB * ngrp_win;
-      for (int i = warp; i < nbias; i += nwarps) {
-        const int b = i / ngrp_win, gl = i - b * ngrp_win;
-        float sum = 0.f;
-        if (b < a.batch) {
-          const uint16_t* xr = a.x + static_cast<int64_t>(b) * a.k + (wgrp0 + gl) * G;
-          for (int e = lane; e < G; e += 32)
-            sum += __bfloat162float(__ushort_as_bfloat16(xr[e]));
+          const uint4* src = reinterpret_cast<const uint4*>(
+              a.x + static_cast<int64_t>(b) * a.k + (wgrp0 + gl) * G + sc * 32);
+          uint4 v[4];
+#pragma unroll
+          for (int c = 0; c < 4; ++c) v[c] = __ldg(src + c);
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            const uint32_t wv[4] = {v[c].x, v[c].y, v[c].z, v[c].w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              xv[8 * c + 2 * e] = __uint_as_float(wv[e] << 16);
+              xv[8 * c + 2 * e + 1] = __uint_as_float(wv[e] & 0xFFFF0000u);
+            }
+          }
+        } else {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) xv[e] = 0.f;
         }
 #pragma unroll
-        for (int o = 16; o >= 1; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-        if (lane == 0)
-          bias[b * wg + gl] = ASYM ? sum * 0x1p-24f : -static_cast<float>(HALF) * 0x1p-24f * sum;
+        for (int e = 0; e < 32; ++e) sum += xv[e];
+        uint32_t pr[NP];
+#pragma unroll
+        for (int p = 0; p < NP; ++p) {
+          int ea, eb;
+          float mult;
+          pair_desc<Q>(p, ea, eb, mult);
+          __half2 hv = __floats2half2_rn(xv[ea] * mult, xv[eb] * mult);
+          pr[p] = *reinterpret_cast<uint32_t*>(&hv);
+        }
+#pragma unroll
+        for (int c = 0; c < NP / 4; ++c)
+          *reinterpret_cast<uint4*>(dst + sc * NP * 4 + 16 * c) =
+              make_uint4(pr[4 * c], pr[4 * c + 1], pr[4 * c + 2], pr[4 * c + 3]);
       }
+      // symmetric: -2^(q-1) * 2^-24 * sum_g x; asymmetric: 2^-24 * sum_g x
+      bias[b * wg + gl] = ASYM ? sum * 0x1p-24f : -static_cast<float>(HALF) * 0x1p-24f * sum;
     }
     __syncthreads();
 
-    // ---- warps interleave over the window's 8-group steps ----
-    for (int64_t step = wstep + warp; step < wsteps_end; step += nwarps) {
-      const int gl0 = static_cast<int>(step * 8 - wgrp0);  // local index of the step's group 0
-      float d[RT][4];
-#pragma unroll
-      for (int tt = 0; tt < RT; ++tt) d[tt][0] = d[tt][1] = d[tt][2] = d[tt][3] = 0.f;
-      float dnb[NB > 1 ? NB : 1][RT][4];
-      if constexpr (NB > 1) {
+    auto compute_unit = [&](const Unit<Q, RT>& U, int u) {
+      const int64_t step = wstep + warp + static_cast<int64_t>(u / SC) * nwarps;
+      const int sc = u % SC;
+      const int gl0 = static_cast<int>(step * 8 - wgrp0);
+      if (sc == 0) {
 #pragma unroll
         for (int b = 0; b < NB; ++b)
 #pragma unroll
-          for (int tt = 0; tt < RT; ++tt)
-            dnb[b][tt][0] = dnb[b][tt][1] = dnb[b][tt][2] = dnb[b][tt][3] = 0.f;
-      }
-      for (int sc = 0; sc < SC; ++sc) {
+          for (int tt = 0; tt < RT; ++tt) d[b][tt][0] = d[b][tt][1] = d[b][tt][2] = d[b][tt][3] = 0.f;
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int grp = static_cast<int>(step * 8) + 2 * tq + h;  // this lane's group
-          const bool gok = grp < nG;
-          uint32_t w[RT][2][NW];
+        for (int tt = 0; tt < RT; ++tt)
 #pragma unroll
-          for (int tt = 0; tt < RT; ++tt)
-#pragma unroll
-            for (int hh = 0; hh < 2; ++hh)
-              load_sub<Q>(rowp[tt][hh], grp, sc, G, gok && rowok[tt][hh], w[tt][hh]);
-          // column gq of B carries group step*8 + gq: active for this h iff
-          // gq == 2*tq + h (the lane whose own group is that column); the
-          // other lanes read a block of zeros
-          const int colgrp = static_cast<int>(step * 8) + gq;
-          const bool active = (gq == 2 * tq + h) && (colgrp < nG);
-          const unsigned char* xp0 =
-              active ? xs + static_cast<size_t>(gl0 + gq) * pitch + sc * NP * 4 : zero;
-          const size_t bstride = active ? static_cast<size_t>(wg) * pitch : 0;
-#pragma unroll
-          for (int j = 0; j < NP / 2; j += 2) {  // two mmas per 16-byte B load
-            uint32_t A[2][RT][4];
-#pragma unroll
-            for (int jj = 0; jj < 2; ++jj) {
-              const int p = 2 * (j + jj);
-#pragma unroll
-              for (int tt = 0; tt < RT; ++tt) {
-                A[jj][tt][0] = unpack_pair<Q>(w[tt][0], p);      // row g,   k 2t..
-                A[jj][tt][1] = unpack_pair<Q>(w[tt][1], p);      // row g+8, k 2t..
-                A[jj][tt][2] = unpack_pair<Q>(w[tt][0], p + 1);  // row g,   k 2t+8..
-                A[jj][tt][3] = unpack_pair<Q>(w[tt][1], p + 1);  // row g+8, k 2t+8..
-              }
-            }
-#pragma unroll
-            for (int b = 0; b < NB; ++b) {
-              const uint4 bv = *reinterpret_cast<const uint4*>(xp0 + b * bstride + j * 8);
-#pragma unroll
-              for (int tt = 0; tt < RT; ++tt) {
-                float(&dd)[4] = (NB == 1) ? d[tt] : dnb[b][tt];
-                mma16816(dd, A[0][tt][0], A[0][tt][1], A[0][tt][2], A[0][tt][3], bv.x, bv.y);
-                mma16816(dd, A[1][tt][0], A[1][tt][1], A[1][tt][2], A[1][tt][3], bv.z, bv.w);
-              }
-            }
+          for (int hh = 0; hh < 2; ++hh) {
+            st[tt][hh] = U.s[tt][hh];
+            mt[tt][hh] = U.m[tt][hh];
           }
-        }
       }
-      // ---- per-group scale (and min) ----
-      const int gA = static_cast<int>(step * 8) + 2 * tq;  // columns 2tq, 2tq+1
 #pragma unroll
-      for (int tt = 0; tt < RT; ++tt) {
+      for (int h = 0; h < 2; ++h) {
+        // column gq of B carries group step*8 + gq; it is this lane's own
+        // group for h iff gq == 2*tq + h.  Other lanes read zeros.
+        const bool active = (gq == 2 * tq + h) && (step * 8 + gq < nG);
+        const unsigned char* xp0 =
+            active ? xs + static_cast<size_t>(gl0 + gq) * pitch + sc * NP * 4 : zero;
+        const size_t bstride = active ? static_cast<size_t>(wg) * pitch : 0;
 #pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-          const int64_t r = row0 + 16 * tt + gq + 8 * hh;
-          float s[2] = {0.f, 0.f}, m[2] = {0.f, 0.f};
+        for (int j = 0; j < NP / 2; j += 2) {  // two mmas per 16-byte B load
+          uint32_t A[2][RT][4];
 #pragma unroll
-          for (int c = 0; c < 2; ++c) {
-            if (rowok[tt][hh] && gA + c < nG) {
-              const int64_t gi = r * gpr + gA + c;
-              s[c] = __half2float(__ushort_as_half(__ldcs(a.scales + gi)));
-              if constexpr (ASYM) m[c] = __half2float(__ushort_as_half(__ldcs(a.mins + gi)));
+          for (int jj = 0; jj < 2; ++jj) {
+            const int p = 2 * (j + jj);
+#pragma unroll
+            for (int tt = 0; tt < RT; ++tt) {
+              A[jj][tt][0] = unpack_pair<Q>(U.w[h][tt][0], p);      // row g,   k 2t..
+              A[jj][tt][1] = unpack_pair<Q>(U.w[h][tt][1], p);      // row g+8, k 2t..
+              A[jj][tt][2] = unpack_pair<Q>(U.w[h][tt][0], p + 1);  // row g,   k 2t+8..
+              A[jj][tt][3] = unpack_pair<Q>(U.w[h][tt][1], p + 1);  // row g+8, k 2t+8..
             }
           }
 #pragma unroll
           for (int b = 0; b < NB; ++b) {
-            const float* dv = (NB == 1) ? d[tt] : dnb[b][tt];
-            const float b0v = (gA < nG) ? bias[b * wg + gl0 + 2 * tq] : 0.f;
-            const float b1v = (gA + 1 < nG) ? bias[b * wg + gl0 + 2 * tq + 1] : 0.f;
-            const float d0 = dv[2 * hh], d1 = dv[2 * hh + 1];
-            if constexpr (ASYM) {
-              acc[b][tt][hh] += s[0] * d0 + m[0] * b0v + s[1] * d1 + m[1] * b1v;
-            } else {
-              acc[b][tt][hh] += s[0] * (d0 + b0v) + s[1] * (d1 + b1v);
+            const uint4 bv = *reinterpret_cast<const uint4*>(xp0 + b * bstride + j * 8);
+#pragma unroll
+            for (int tt = 0; tt < RT; ++tt) {
+              mma16816(d[b][tt], A[0][tt][0], A[0][tt][1], A[0][tt][2], A[0][tt][3], bv.x, bv.y);
+              mma16816(d[b][tt], A[1][tt][0], A[1][tt][1], A[1][tt][2], A[1][tt][3], bv.z, bv.w);
             }
           }
         }
+      }
+      if (sc == SC - 1) {
+        // per-group scale (and min): lane holds columns 2tq, 2tq+1 = its groups
+        const int gl = gl0 + 2 * tq;
+        const bool ok0 = step * 8 + 2 * tq < nG, ok1 = step * 8 + 2 * tq + 1 < nG;
+#pragma unroll
+        for (int tt = 0; tt < RT; ++tt)
+#pragma unroll
+          for (int hh = 0; hh < 2; ++hh) {
+            const __half2 s2 = *reinterpret_cast<const __half2*>(&st[tt][hh]);
+            const float2 sf = __half22float2(s2);
+            float2 mf = make_float2(0.f, 0.f);
+            if constexpr (ASYM) mf = __half22float2(*reinterpret_cast<const __half2*>(&mt[tt][hh]));
+#pragma unroll
+            for (int b = 0; b < NB; ++b) {
+              const float b0v = ok0 ? bias[b * wg + gl] : 0.f;
+              const float b1v = ok1 ? bias[b * wg + gl + 1] : 0.f;
+              const float d0 = d[b][tt][2 * hh], d1 = d[b][tt][2 * hh + 1];
+              if constexpr (ASYM) {
+                acc[b][tt][hh] += sf.x * d0 + mf.x * b0v + sf.y * d1 + mf.y * b1v;
+              } else {
+                acc[b][tt][hh] += sf.x * (d0 + b0v) + sf.y * (d1 + b1v);
+              }
+            }
+          }
+      }
+    };
+
+    // ---- ping-pong over this warp's units: loads run one unit ahead ----
+    auto unit_step = [&](int64_t uu) { return wstep + warp + (uu / SC) * nwarps; };
+    for (int u = 0; u < nunits; u += 2) {
+      if (u + 1 < nunits) load_unit(ub, unit_step(u + 1), (u + 1) % SC);
+      compute_unit(ua, u);
+      if (u + 1 < nunits) {
+        if (u + 2 < nunits) load_unit(ua, unit_step(u + 2), (u + 2) % SC);
+        compute_unit(ub, u + 1);
       }
     }
   }
@@ -434,10 +491,11 @@ Plan make_plan(const sss_qtensor_t& t, int batch) {
   p.ks = static_cast<int>((nsteps + p.steps_per_cta - 1) / p.steps_per_cta);
   if (p.ks < 1) p.ks = 1;
   p.warps = std::max(1, std::min(kMaxWarps, p.steps_per_cta));
-  const int win_base = (p.nb == 1) ? kWindowGroups : std::max(8, 64 / p.nb);
-  p.window_groups = static_cast<int>(std::min<int64_t>(win_base, static_cast<int64_t>(p.steps_per_cta) * 8));
-  p.window_groups = (p.window_groups + 7) / 8 * 8;
   const int pitch = pitch_bytes(t.q, t.group);
+  // stage as much of the CTA's k-range as fits in ~48 KB, in whole steps
+  int win = static_cast<int>((48 * 1024) / (static_cast<int64_t>(p.nb) * pitch)) / 8 * 8;
+  win = std::max(8, win);
+  p.window_groups = static_cast<int>(std::min<int64_t>(win, static_cast<int64_t>(p.steps_per_cta) * 8));
   p.smem = static_cast<size_t>(p.nb) * p.window_groups * pitch + 128 +
            sizeof(float) * (static_cast<size_t>(p.nb) * p.window_groups +
                             static_cast<size_t>(p.warps) * p.nb * p.rt * 16 +

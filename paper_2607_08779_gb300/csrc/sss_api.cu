@@ -64,6 +64,20 @@ cudaError_t ensure_smem_impl(const void* kernel, int bytes) {
   return e;
 }
 
+EncodeTiledFn tensor_map_encoder() {
+  static std::once_flag once;
+  static EncodeTiledFn fn = nullptr;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
 int device_sm_count() {
   static std::mutex mu;
   static int cache[64] = {0};
@@ -113,7 +127,7 @@ sss_status_t sss_quantize(const float* w, const sss_qtensor_t* out,
   if (w == nullptr) return SSS_E_ARG;
   if (!aligned(w, 16)) return SSS_E_ALIGN;
   if (!aligned(out->scales, 2) || (out->mins && !aligned(out->mins, 2))) return SSS_E_ALIGN;
-  if (out->q == 4 && !aligned(out->codes, 2)) return SSS_E_ALIGN;
+  if (!aligned(out->codes, 16)) return SSS_E_ALIGN;
   if (dev_status && !aligned(dev_status, 4)) return SSS_E_ALIGN;
   return finish("sss_quantize",
                 launch_quantize(w, *out, clip_counts, dev_status,
@@ -161,8 +175,44 @@ sss_status_t sss_gemv(const sss_qtensor_t* qt, const uint16_t* x_bf16, int32_t b
                   cudaMemsetAsync(y, 0, sizeof(float) * static_cast<size_t>(batch) * qt->n,
                                   static_cast<cudaStream_t>(stream)));
   }
+  if (batch == 1 && gemv_stream_eligible(*qt, x_bf16)) {
+    const sss_qtensor_t* one[1] = {qt};
+    float* yy[1] = {y};
+    return finish("sss_gemv", launch_gemv_stream(one, yy, 1, x_bf16, 0u, dev_status,
+                                                 static_cast<cudaStream_t>(stream)));
+  }
   return finish("sss_gemv", launch_gemv(*qt, x_bf16, batch, y, workspace,
                                         static_cast<cudaStream_t>(stream)));
+}
+
+sss_status_t sss_gemv_multi(const sss_qtensor_t* const* qts, float* const* ys, int32_t count,
+                            const uint16_t* x_bf16, uint32_t flags, uint32_t* dev_status,
+                            void* stream) {
+  if (qts == nullptr || ys == nullptr || count < 1 || count > 4) return SSS_E_ARG;
+  if ((flags & ~(SSS_GEMV_PDL | SSS_GEMV_WEIGHTS_READY)) != 0) return SSS_E_ARG;
+  bool stream_ok = true;
+  for (int j = 0; j < count; ++j) {
+    sss_status_t st = check_tensor(qts[j]);
+    if (st != SSS_OK) return st;
+    const sss_qtensor_t& t = *qts[j];
+    const sss_qtensor_t& t0 = *qts[0];
+    if (t.k != t0.k || t.q != t0.q || t.group != t0.group || t.grid != t0.grid) return SSS_E_ARG;
+    if (t.n > 0 && ys[j] == nullptr) return SSS_E_ARG;
+    if (ys[j] != nullptr && !aligned(ys[j], 4)) return SSS_E_ALIGN;
+    if (t.n > 0 && !gemv_stream_eligible(t, x_bf16)) stream_ok = false;
+    if (t.n == 0) stream_ok = false;
+  }
+  if (x_bf16 == nullptr) return SSS_E_ARG;
+  if (dev_status && !aligned(dev_status, 4)) return SSS_E_ALIGN;
+  if (stream_ok && qts[0]->k > 0) {
+    return finish("sss_gemv_multi", launch_gemv_stream(qts, ys, count, x_bf16, flags, dev_status,
+                                                       static_cast<cudaStream_t>(stream)));
+  }
+  for (int j = 0; j < count; ++j) {
+    sss_status_t st = sss_gemv(qts[j], x_bf16, 1, ys[j], nullptr, 0, dev_status, stream);
+    if (st != SSS_OK) return st;
+  }
+  return SSS_OK;
 }
 
 sss_status_t sss_gemm(const sss_qtensor_t* qt, const uint16_t* x_bf16, int64_t m,

@@ -2,6 +2,7 @@
 // the library (not installed; the public interface is include/sss.h).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
@@ -14,6 +15,14 @@ namespace sss {
 // Number of SMs of the current device (queried once per device).
 int device_sm_count();
 
+// cuTensorMapEncodeTiled, resolved through the runtime's driver entry point
+// (the library does not link libcuda); nullptr if unavailable.
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn tensor_map_encoder();
+
 // Launchers.  Arguments are validated by the C ABI before these run.
 cudaError_t launch_quantize(const float* w, const sss_qtensor_t& t,
                             uint8_t* clip_counts, uint32_t* status,
@@ -24,6 +33,11 @@ cudaError_t launch_dequantize(const sss_qtensor_t& t, void* out, int out_dtype,
 size_t gemv_workspace_bytes(const sss_qtensor_t& t, int batch);
 cudaError_t launch_gemv(const sss_qtensor_t& t, const uint16_t* x, int batch,
                         float* y, void* workspace, cudaStream_t stream);
+
+bool gemv_stream_eligible(const sss_qtensor_t& t, const uint16_t* x);
+cudaError_t launch_gemv_stream(const sss_qtensor_t* const* ts, float* const* ys, int count,
+                               const uint16_t* x, uint32_t flags, uint32_t* status,
+                               cudaStream_t stream);
 
 size_t gemm_workspace_bytes(const sss_qtensor_t& t, int64_t m);
 cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m,

@@ -31,7 +31,10 @@ STATUS_NAMES = {0: "SSS_OK", 1: "SSS_E_ARG", 2: "SSS_E_UNSUPPORTED", 3: "SSS_E_A
                 4: "SSS_E_CUDA", 5: "SSS_E_WORKSPACE"}
 
 EXPORTS = ("sss_codes_bytes", "sss_status_string", "sss_last_error", "sss_quantize",
-           "sss_dequantize", "sss_gemv", "sss_gemm", "sss_workspace_bytes")
+           "sss_dequantize", "sss_gemv", "sss_gemv_multi", "sss_gemm", "sss_workspace_bytes")
+
+GEMV_PDL = 0x1
+GEMV_WEIGHTS_READY = 0x2
 
 
 class SssError(RuntimeError):
@@ -89,6 +92,9 @@ def load(build_if_needed: bool = True):
         L.sss_dequantize.restype = i32
         L.sss_gemv.argtypes = [P, vp, i32, vp, vp, sz, vp, vp]
         L.sss_gemv.restype = i32
+        L.sss_gemv_multi.argtypes = [ctypes.POINTER(P), ctypes.POINTER(vp), i32, vp,
+                                     ctypes.c_uint32, vp, vp]
+        L.sss_gemv_multi.restype = i32
         L.sss_gemm.argtypes = [P, vp, i64, vp, vp, sz, vp, vp]
         L.sss_gemm.restype = i32
         L.sss_workspace_bytes.argtypes = [P, i64, i32]
@@ -204,6 +210,21 @@ def sss_gemv(qt: QTensor, x, y=None, workspace=None, dev_status=None, stream=Non
                          _ptr(dev_status), _stream(stream))
     _check("sss_gemv", st)
     return y
+
+
+def sss_gemv_multi(qts, x, ys=None, flags: int = 0, dev_status=None, stream=None):
+    """y_j [n_j] fp32 = x [k] (bf16) @ dequant(qt_j)^T for 1..4 matrices sharing x."""
+    import torch
+
+    if ys is None:
+        ys = [torch.empty((qt.n,), dtype=torch.float32, device=x.device) for qt in qts]
+    descs = [qt.desc() for qt in qts]
+    parr = (ctypes.POINTER(QTensorDesc) * len(qts))(*[ctypes.pointer(d) for d in descs])
+    yarr = (ctypes.c_void_p * len(qts))(*[_ptr(y) for y in ys])
+    st = load().sss_gemv_multi(parr, yarr, len(qts), _ptr(x), flags, _ptr(dev_status),
+                               _stream(stream))
+    _check("sss_gemv_multi", st)
+    return ys
 
 
 def sss_gemm(qt: QTensor, x, y=None, workspace=None, dev_status=None, stream=None):

@@ -1,0 +1,95 @@
+"""Parity of the streaming batch-1 GEMV (sss_gemv_multi and the batch-1
+sss_gemv path) with the fp64 oracle, for single and fused multi-matrix
+launches, with and without programmatic dependent launch."""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2607_08779_gb300 import inputs, sss
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+from gpu_util import REL_TOL, qtensor_from_oracle, rel_err_per_row, to_dev, x_bits  # noqa: E402
+
+QS = (2, 3, 4)
+GRIDS = (sss.GRID_UNSIGNED_SYM, sss.GRID_SIGNED_SYM, sss.GRID_ASYM)
+
+
+def make(n, k, q, g, grid, seed):
+    W = inputs.student_t_weights(n, k, seed)
+    codes, scales, mins, _, _ = oracle.quantize(W, q, g, grid)
+    return qtensor_from_oracle(codes, scales, mins, n, k, q, g, grid), (codes, scales, mins)
+
+
+def check_multi(ns, k, q, g, grid, seed, flags=0):
+    mats = [make(n, k, q, g, grid, seed + 31 * i) for i, n in enumerate(ns)]
+    xb = x_bits(1, k, seed + 7)
+    x = to_dev(xb[0].view(np.int16)).view(torch.bfloat16)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ys = sss.sss_gemv_multi([m[0] for m in mats], x, flags=flags, dev_status=status)
+    ys2 = sss.sss_gemv_multi([m[0] for m in mats], x, flags=flags)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    worst = 0.0
+    for (qt, (codes, scales, mins)), y, y2, n in zip(mats, ys, ys2, ns):
+        assert torch.equal(y, y2), "not deterministic"
+        yref = oracle.gemv(codes, scales, mins, n, k, q, g, grid, xb)
+        err = rel_err_per_row(y.cpu().numpy()[None, :], yref)
+        assert err.max() <= REL_TOL, f"rel err {err.max():.3e}"
+        worst = max(worst, float(err.max()))
+    return worst
+
+
+@pytest.mark.parametrize("grid", GRIDS)
+@pytest.mark.parametrize("q", QS)
+@pytest.mark.parametrize("g", [32, 64, 128])
+def test_stream_single_ragged_rows(q, g, grid):
+    # 100 rows: a ragged last tile; k = 2048 (8 units of 256 codes)
+    check_multi([100], 2048, q, g, grid, q * 10 + g + grid)
+
+
+@pytest.mark.parametrize("q", QS)
+def test_stream_fused_three(q):
+    """q/k/v-shaped fusion at reduced rows: three matrices, one x."""
+    check_multi([512, 128, 128], 4096, q, 32, sss.GRID_SIGNED_SYM, 40 + q)
+
+
+@pytest.mark.parametrize("flags", [0, sss.GEMV_PDL, sss.GEMV_PDL | sss.GEMV_WEIGHTS_READY])
+def test_stream_flags(flags):
+    check_multi([300, 77], 1024, 4, 32, sss.GRID_SIGNED_SYM, 9, flags=flags)
+
+
+@pytest.mark.parametrize("grid", GRIDS)
+def test_stream_llama_qkv_and_gate_up(grid):
+    n_q, k = inputs.LLAMA3_8B_LAYER["q_proj"]
+    check_multi([n_q, 1024, 1024], k, 4, 32, grid, 3)
+    check_multi([14336, 14336], 4096, 4, 32, grid, 4)
+
+
+@pytest.mark.parametrize("q", QS)
+def test_stream_down_proj_long_k(q):
+    n, k = inputs.LLAMA3_8B_LAYER["down_proj"]
+    check_multi([n], k, q, 32, sss.GRID_SIGNED_SYM, 5 + q)
+
+
+def test_stream_small_rows_many_tiles():
+    check_multi([1, 17, 16, 33], 256, 4, 32, sss.GRID_SIGNED_SYM, 12)
+
+
+def test_multi_fallback_shapes():
+    """k not a multiple of 256: the multi entry falls back to per-matrix GEMVs."""
+    check_multi([70, 9], 96, 4, 32, sss.GRID_ASYM, 13)
+    check_multi([70], 1024 + 128, 3, 128, sss.GRID_SIGNED_SYM, 14)
+
+
+def test_stream_precision_far_inside_gate():
+    assert check_multi([2048], 4096, 4, 32, sss.GRID_SIGNED_SYM, 15) < 2e-5
+
+
+def test_multi_rejects_mixed_shapes():
+    a, _ = make(64, 256, 4, 32, sss.GRID_SIGNED_SYM, 1)
+    b, _ = make(64, 512, 4, 32, sss.GRID_SIGNED_SYM, 2)
+    x = torch.zeros(256, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(sss.SssError):
+        sss.sss_gemv_multi([a, b], x)
