@@ -13,8 +13,8 @@
  *
  * Conventions for every entry point:
  *  - All tensor pointers are DEVICE pointers owned by the caller.  No entry
- *    point allocates device memory (sss_gemm keeps a small per-device cache
- *    of encoded tensor maps in host memory).
+ *    point allocates device memory; the library keeps only small host-side
+ *    per-device records (SM count, raised shared-memory limits of kernels).
  *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
  *    stream).  Every call is asynchronous on that stream; none synchronises.
  *  - The return value reports synchronous argument checks and launch errors.
@@ -71,8 +71,8 @@ typedef enum {
                                    for symmetric grids, u = 0 and s = +0 for ASYM)     */
 #define SSS_FLAG_RANGE 0x2u     /* a stored fp16 scale or min is infinite (|s| >= 65520),
                                    or the fp32 ASYM step overflowed (codes then 0)     */
-#define SSS_FLAG_TIMEOUT 0x4u   /* a bounded pipeline wait in sss_gemm expired; the
-                                   output is incomplete                               */
+#define SSS_FLAG_TIMEOUT 0x4u   /* a bounded pipeline wait (sss_gemm, or the batch-1
+                                   streaming GEMV) expired; the output is incomplete  */
 
 typedef enum { SSS_OUT_F32 = 0, SSS_OUT_F16 = 1, SSS_OUT_BF16 = 2 } sss_dtype_t;
 

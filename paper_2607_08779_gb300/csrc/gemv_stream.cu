@@ -46,6 +46,7 @@ constexpr int kThreads = kWarps * 32;
 constexpr int kMaxJobs = 4;
 constexpr uint64_t kWaitNs = 1000000000ull;
 
+
 template <int Q>
 struct SQ;
 template <>
@@ -228,26 +229,32 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   // allow the next kernel in the stream to be scheduled as SMs free up
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-  // ---- this warp's stream: tiles t = (blockIdx.x * ngrp + grp) + i * (gridDim.x
-  // * ngrp), i = 0, 1, ..., and in each tile the units u = kw, kw + KW, ... ----
+  // ---- this warp's stream: tiles t = (i * ngrp + grp) * gridDim.x + blockIdx.x,
+  // i = 0, 1, ... (consecutive tiles go to different SMs, so every SM gets
+  // within one tile of the same work), and in each tile the units u = kw,
+  // kw + KW, ... ----
   const int64_t tstride = static_cast<int64_t>(gridDim.x) * ngrp;
-  const int64_t tfirst = static_cast<int64_t>(blockIdx.x) * ngrp + grp;
+  const int64_t tfirst = static_cast<int64_t>(grp) * gridDim.x + blockIdx.x;
   const int64_t my_tiles = tfirst < a.ntiles ? (a.ntiles - tfirst + tstride - 1) / tstride : 0;
   const bool has_units = kw < nunits;
 
   // This warp's flat unit stream: unit k is unit u = kw + (k % upw) * KW of
-  // its i = k / upw-th tile, upw = units per tile for this warp.
+  // its i = k / upw-th tile, upw = units per tile for this warp (the host
+  // keeps every count below 2^31).
   const int upw = has_units ? (nunits - kw + KW - 1) >> lgkw : 0;
-  const int64_t total = my_tiles * upw;
+  const int total = static_cast<int>(my_tiles) * upw;
 
-  // fetch cursor: tile index, unit, and that tile's row pointers
-  int64_t fi = 0;
-  int fu = kw;
-  const uint8_t* frow[2] = {nullptr, nullptr};
-  const uint16_t* fsrow[2] = {nullptr, nullptr};
-  const uint16_t* fmrow[2] = {nullptr, nullptr};
-  auto set_tile = [&](int64_t i) {
-    if (i >= my_tiles) return;
+  constexpr int UB = 32 * Q;    // code bytes of one row in one unit
+  constexpr int SPU = 256 / G;  // scales of one row in one unit
+  // the lane's byte offset in a unit's codes (sub-chunks 2tq, 2tq+1; q=3
+  // addresses its planes per sub-chunk below) and its scale index in the
+  // unit: the pair of groups 2tq, 2tq+1 for g=32, else its one group
+  const int lane_c = Q == 4 ? 32 * tq : (Q == 2 ? 16 * tq : 0);
+  const int lane_s = G == 32 ? 2 * tq : (G == 64 ? tq : (tq >> 1));
+
+  // the code/scale/min pointers of rows g and g+8 of this warp's i-th tile,
+  // at its first unit
+  auto tile_ptrs = [&](int64_t i, const uint8_t** c, const uint16_t** sc, const uint16_t** mn) {
     const int64_t t = tfirst + i * tstride;
     int j = 0;
     while (j + 1 < a.njobs && t >= a.job[j + 1].tile0) ++j;
@@ -257,37 +264,47 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
     for (int hh = 0; hh < 2; ++hh) {
       int64_t r = row0 + gq + 8 * hh;
       if (r >= jb.n) r = jb.n - 1;  // a valid row; results past n are never stored
-      frow[hh] = jb.codes + r * row_bytes;
-      fsrow[hh] = jb.scales + r * nG;
-      if constexpr (ASYM) fmrow[hh] = jb.mins + r * nG;
+      c[hh] = jb.codes + r * row_bytes + kw * UB + lane_c;
+      sc[hh] = jb.scales + r * nG + kw * SPU + lane_s;
+      if constexpr (ASYM) mn[hh] = jb.mins + r * nG + kw * SPU + lane_s;
     }
   };
+  // fetch cursor: the next unit to load into registers
+  int64_t fi = 0;
+  int fleft = 0;
+  const uint8_t* cp[2] = {nullptr, nullptr};
+  const uint16_t* sp[2] = {nullptr, nullptr};
+  const uint16_t* mp[2] = {nullptr, nullptr};
+  auto set_tile = [&](int64_t i) {
+    if (i >= my_tiles) return;
+    tile_ptrs(i, cp, sp, mp);
+    fleft = upw;
+  };
   // the registers of one unit: code words of (row half hh, column parity h),
-  // and the aligned fp16 scale (min) pair of each row
+  // and the fp16 scale (min) of each row: the pair of the lane's two groups
+  // for g=32, else its one group in the low half
   struct Regs {
     uint32_t w[2][2][4];
     uint32_t s[2], m[2];
   };
   auto fetch = [&](Regs& rg) {
-    if (fi >= my_tiles) return;
-    const int s0 = fu * 8 + 2 * tq;  // the lane's first sub-chunk (column 2tq)
 #pragma unroll
     for (int hh = 0; hh < 2; ++hh) {
-      const uint8_t* rp = frow[hh];
-      if constexpr (Q == 4) {  // sub-chunk s at byte 16s
+      const uint8_t* rp = cp[hh];
+      if constexpr (Q == 4) {  // sub-chunk 2tq + h at byte 32tq + 16h
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-          const uint4 v = __ldcs(reinterpret_cast<const uint4*>(rp + 16 * (s0 + h)));
+          const uint4 v = __ldcs(reinterpret_cast<const uint4*>(rp + 16 * h));
           rg.w[hh][h][0] = v.x; rg.w[hh][h][1] = v.y; rg.w[hh][h][2] = v.z; rg.w[hh][h][3] = v.w;
         }
-      } else if constexpr (Q == 2) {  // sub-chunks s0, s0+1 at bytes 8s: 16 contiguous bytes
-        const uint4 v = __ldcs(reinterpret_cast<const uint4*>(rp + 8 * s0));
+      } else if constexpr (Q == 2) {  // sub-chunks 2tq, 2tq+1: 16 contiguous bytes
+        const uint4 v = __ldcs(reinterpret_cast<const uint4*>(rp));
         rg.w[hh][0][0] = v.x; rg.w[hh][0][1] = v.y;
         rg.w[hh][1][0] = v.z; rg.w[hh][1][1] = v.w;
       } else {  // q=3: two low-plane words and one high-plane word per sub-chunk
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-          const int e0 = (s0 + h) * 32;
+          const int e0 = (2 * tq + h) * 32;  // within the unit (units hold whole groups)
           const int gbyte = (e0 >> LGG) * (3 * G / 8);
           const int sc = (e0 & (G - 1)) >> 5;
           const uint32_t* lo = reinterpret_cast<const uint32_t*>(rp + gbyte + 8 * sc);
@@ -296,16 +313,18 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
           rg.w[hh][h][2] = __ldcs(reinterpret_cast<const uint32_t*>(rp + gbyte + G / 4 + 4 * sc));
         }
       }
-      const int gpair = ((s0 << 5) >> LGG) & ~1;
-      rg.s[hh] = __ldcs(reinterpret_cast<const uint32_t*>(fsrow[hh] + gpair));
-      if constexpr (ASYM) rg.m[hh] = __ldcs(reinterpret_cast<const uint32_t*>(fmrow[hh] + gpair));
+      if constexpr (G == 32) {
+        rg.s[hh] = __ldcs(reinterpret_cast<const uint32_t*>(sp[hh]));
+        if constexpr (ASYM) rg.m[hh] = __ldcs(reinterpret_cast<const uint32_t*>(mp[hh]));
+      } else {
+        rg.s[hh] = __ldcs(reinterpret_cast<const unsigned short*>(sp[hh]));
+        if constexpr (ASYM) rg.m[hh] = __ldcs(reinterpret_cast<const unsigned short*>(mp[hh]));
+      }
+      cp[hh] += UB * KW;
+      sp[hh] += SPU * KW;
+      if constexpr (ASYM) mp[hh] += SPU * KW;
     }
-    fu += KW;
-    if (fu >= nunits) {
-      fu = kw;
-      ++fi;
-      set_tile(fi);
-    }
+    if (--fleft == 0) set_tile(++fi);
   };
 
   Regs ring[D];
@@ -354,10 +373,21 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
 
   bool ok = true;
   float acc[2] = {0.f, 0.f};
-  int64_t ci = 0;   // tile of the unit being computed
-  int cu = kw;      // the unit
+  // column gq of B carries the lane's sub-chunk 8u + gq in the mma of parity
+  // h only when it is the sub-chunk of this quad's own A rows (gq == 2tq + h);
+  // otherwise the lane reads zeros
+  const bool act0 = gq == 2 * tq, act1 = gq == 2 * tq + 1;
+  const unsigned char* xl = nullptr;  // the lane's B data of the unit being computed
+  const float* bl = nullptr;          // the sums of its two columns' sub-chunks
+  int cleft = 0;
+  int64_t ci = 0;
+  auto start_tile = [&]() {
+    xl = xs + static_cast<size_t>(kw * 8 + gq) * SL::XPITCH;
+    bl = bias + kw * 8 + 2 * tq;
+    cleft = upw;
+  };
+  start_tile();
   auto compute = [&](const Regs& rg) {
-    const int u = cu;
     // h=0 mmas only write even columns and h=1 mmas odd ones: the lane's
     // column 2tq is in dh[0] and 2tq+1 in dh[1]
     float dh[2][4];
@@ -365,10 +395,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
     for (int h = 0; h < 2; ++h) dh[h][0] = dh[h][1] = dh[h][2] = dh[h][3] = 0.f;
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      // column gq of B carries sub-chunk u*8 + gq: active for this h iff it
-      // is this lane's own sub-chunk (gq == 2tq + h); others read zeros
-      const unsigned char* xp =
-          (gq == 2 * tq + h) ? xs + static_cast<size_t>(u * 8 + gq) * SL::XPITCH : zero;
+      const unsigned char* xp = (h ? act1 : act0) ? xl : zero;
 #pragma unroll
       for (int jm = 0; jm < NP / 2; jm += 2) {
         const uint4 bv = *reinterpret_cast<const uint4*>(xp + jm * 8);
@@ -381,23 +408,32 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
         }
       }
     }
-    // per-group scale (and min) of this lane's two columns
-    const int s0 = u * 8 + 2 * tq;
-    const int sel0 = ((s0 << 5) >> LGG) & 1, sel1 = (((s0 + 1) << 5) >> LGG) & 1;
-    const float bb0 = bias[s0], bb1 = bias[s0 + 1];
+    const float2 bb = *reinterpret_cast<const float2*>(bl);
 #pragma unroll
     for (int hh = 0; hh < 2; ++hh) {
-      const float2 sf = __half22float2(*reinterpret_cast<const __half2*>(&rg.s[hh]));
-      const float s_0 = sel0 ? sf.y : sf.x;
-      const float s_1 = sel1 ? sf.y : sf.x;
+      float s_0, s_1, m_0 = 0.f, m_1 = 0.f;
+      if constexpr (G == 32) {
+        const float2 sf = __half22float2(*reinterpret_cast<const __half2*>(&rg.s[hh]));
+        s_0 = sf.x;
+        s_1 = sf.y;
+        if constexpr (ASYM) {
+          const float2 mf = __half22float2(*reinterpret_cast<const __half2*>(&rg.m[hh]));
+          m_0 = mf.x;
+          m_1 = mf.y;
+        }
+      } else {
+        s_0 = s_1 = __half2float(__ushort_as_half(static_cast<unsigned short>(rg.s[hh])));
+        if constexpr (ASYM) m_0 = m_1 = __half2float(__ushort_as_half(static_cast<unsigned short>(rg.m[hh])));
+      }
       const float d0 = dh[0][2 * hh], d1 = dh[1][2 * hh + 1];
       if constexpr (ASYM) {
-        const float2 mf = __half22float2(*reinterpret_cast<const __half2*>(&rg.m[hh]));
-        acc[hh] += s_0 * d0 + (sel0 ? mf.y : mf.x) * bb0 + s_1 * d1 + (sel1 ? mf.y : mf.x) * bb1;
+        acc[hh] += s_0 * d0 + m_0 * bb.x + s_1 * d1 + m_1 * bb.y;
       } else {
-        acc[hh] += s_0 * (d0 + bb0) + s_1 * (d1 + bb1);
+        acc[hh] += s_0 * (d0 + bb.x) + s_1 * (d1 + bb.y);
       }
     }
+    xl += static_cast<size_t>(8 * SL::XPITCH) * KW;
+    bl += 8 * KW;
   };
   auto tile_end = [&](int64_t i) {
     const int64_t t = tfirst + i * tstride;
@@ -456,18 +492,17 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   }
   // the units, D at a time so the register ring is indexed at compile time;
   // unit k + D - 1 is loaded while unit k is computed
-  for (int64_t k0 = 0; k0 < total; k0 += D) {
+  for (int k0 = 0; k0 < total; k0 += D) {
 #pragma unroll
     for (int r = 0; r < D; ++r) {
-      const int64_t k = k0 + r;
+      const int k = k0 + r;
       if (k < total) {
         if (k + D - 1 < total) fetch(ring[(r + D - 1) % D]);
         compute(ring[r]);
-        cu += KW;
-        if (cu >= nunits) {
+        if (--cleft == 0) {
           tile_end(ci);
-          cu = kw;
           ++ci;
+          start_tile();
         }
       }
     }
@@ -507,7 +542,7 @@ cudaError_t launch_d(StreamArgs& a, int grid, bool pdl, cudaStream_t stream) {
 template <int Q, bool ASYM, int G>
 cudaError_t launch_g(StreamArgs& a, int grid, bool pdl, cudaStream_t stream) {
   if (smem_bytes<Q, ASYM>(a.k, 0) > 227 * 1024) return cudaErrorNotSupported;
-  return launch_d<Q, ASYM, G, (Q == 3 ? 3 : 4)>(a, grid, pdl, stream);
+  return launch_d<Q, ASYM, G, 2>(a, grid, pdl, stream);
 }
 
 template <int Q, bool ASYM>
@@ -519,28 +554,27 @@ cudaError_t launch_q(const sss_qtensor_t* const* ts, StreamArgs& a, bool pdl,
     tiles += (ts[j]->n + 15) / 16;
   }
   a.ntiles = tiles;
-  // Warps per tile: the power of two that minimises the busiest warp's
-  // units (rounds of tiles x units per warp per tile), preferring fewer
-  // warps per tile (less reduction) on ties.
+  // One CTA per SM (fewer when there are fewer tiles); CTA c takes tiles
+  // c, c + grid, ...  Warps per tile: the power of two that minimises the
+  // busiest warp's units (rounds of that CTA's tiles x units per warp per
+  // tile), preferring fewer warps per tile (less reduction) on ties.
   const int sms = device_sm_count();
   const int64_t nunits = a.k / 256;
+  const int grid = static_cast<int>(std::min<int64_t>(sms, tiles));
+  const int64_t per_cta = (tiles + grid - 1) / grid;
   int best = 0;
   int64_t best_cost = INT64_MAX;
   for (int lg = 0; lg <= 4; ++lg) {
     const int kwn = 1 << lg;
     if (kwn > 1 && kwn > nunits) break;
-    const int64_t inflight = static_cast<int64_t>(sms) * (kWarps >> lg);
-    const int64_t rounds = (tiles + inflight - 1) / inflight;
-    const int64_t cost = rounds * ((nunits + kwn - 1) / kwn);
+    const int64_t ngrp = kWarps >> lg;
+    const int64_t cost = ((per_cta + ngrp - 1) / ngrp) * ((nunits + kwn - 1) / kwn);
     if (cost < best_cost) {
       best_cost = cost;
       best = lg;
     }
   }
   a.lgkw = best;
-  const int64_t per_cta = kWarps >> best;
-  const int grid = static_cast<int>(std::max<int64_t>(
-      1, std::min<int64_t>(sms, (tiles + per_cta - 1) / per_cta)));
   switch (ts[0]->group) {
     case 32: return launch_g<Q, ASYM, 32>(a, grid, pdl, stream);
     case 64: return launch_g<Q, ASYM, 64>(a, grid, pdl, stream);
@@ -555,14 +589,14 @@ bool gemv_stream_eligible(const sss_qtensor_t& t, const uint16_t* x) {
   auto al = [](const void* p, size_t b) { return (reinterpret_cast<uintptr_t>(p) % b) == 0; };
   if (t.k <= 0 || t.n <= 0) return false;
   if (t.k % 256 != 0) return false;             // whole 256-code units per row
+  if (((t.n + 15) / 16) * (t.k / 256) >= (int64_t{1} << 29)) return false;  // 32-bit unit counts
   if ((t.k / t.group) % 2 != 0) return false;   // 4-byte scale pairs
   if (!al(t.codes, 16) || !al(t.scales, 4) || !al(x, 16)) return false;
   if (t.grid == SSS_GRID_ASYM && !al(t.mins, 4)) return false;
-  // the staged activations and a 3-deep ring must fit in shared memory
+  // the staged activations must fit in shared memory
   const int64_t nsc = t.k / 32;
   const int64_t xbytes = nsc * ((t.q == 3 ? 32 : 16) * 4 + 16 + 4);
-  const int64_t slot = (2 * 2 * (t.q == 3 ? 3 : (t.q == 4 ? 4 : 2)) + 2 * (t.grid == SSS_GRID_ASYM ? 2 : 1)) * 128;
-  return xbytes + 3 * kWarps * slot + 2048 <= 227 * 1024;
+  return xbytes + 4096 <= 227 * 1024;
 }
 
 cudaError_t launch_gemv_stream(const sss_qtensor_t* const* ts, float* const* ys, int count,

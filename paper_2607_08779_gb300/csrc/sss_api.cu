@@ -93,6 +93,10 @@ int device_sm_count() {
   return cache[dev];
 }
 
+void set_error_message(const char* msg) {
+  snprintf(g_last_error, sizeof g_last_error, "%s", msg);
+}
+
 }  // namespace sss
 
 using namespace sss;

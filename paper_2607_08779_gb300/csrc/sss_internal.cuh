@@ -44,6 +44,9 @@ cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m,
                         float* y, void* workspace, uint32_t* status,
                         cudaStream_t stream);
 
+// Record a message for sss_last_error() on this thread.
+void set_error_message(const char* msg);
+
 // Raise a kernel's dynamic shared-memory limit once per (kernel, device)
 // (the call is not stream-ordered; doing it once keeps launches cheap and
 // capturable in CUDA graphs).
