@@ -210,6 +210,28 @@ sss_status_t sss_gemm(const sss_qtensor_t* qt, const uint16_t* x_bf16,
 size_t sss_workspace_bytes(const sss_qtensor_t* qt, int64_t m_or_batch,
                            int32_t op);
 
+/*
+ * sss_gemm_noalloc -- sss_gemm with its scratch (the fp16 copy of X, m*k*2
+ * bytes) in a static 32 MiB device array of the library instead of a
+ * caller workspace.  The paper has no counterpart: this is a library
+ * convenience for callers that cannot allocate device memory when they
+ * call, e.g. a plain C host with no device allocator, or a serving loop
+ * that must not call cudaMalloc (it synchronises the device and can fail
+ * under memory pressure).  Nothing is allocated at call time.
+ *   Arguments, layouts and errors as sss_gemm, without workspace/ws_bytes.
+ *   Limit: m * k * 2 <= sss_gemm_noalloc_max_scratch_bytes() (33554432);
+ *          larger calls return SSS_E_WORKSPACE (sss_last_error() says why).
+ *   The first call on each device looks up the array's device address with
+ *   that device current (set-up); make that first call before any stream
+ *   capture begins.  Nothing in the scratch needs to start at zero.
+ *   All calls on a device share the one array: calls that overlap in time
+ *   (other streams, other host threads) race on it; callers serialise them.
+ */
+sss_status_t sss_gemm_noalloc(const sss_qtensor_t* qt, const uint16_t* x_bf16,
+                              int64_t m, float* y, uint32_t* dev_status,
+                              void* stream);
+size_t sss_gemm_noalloc_max_scratch_bytes(void);
+
 #ifdef __cplusplus
 }
 #endif

@@ -31,7 +31,8 @@ STATUS_NAMES = {0: "SSS_OK", 1: "SSS_E_ARG", 2: "SSS_E_UNSUPPORTED", 3: "SSS_E_A
                 4: "SSS_E_CUDA", 5: "SSS_E_WORKSPACE"}
 
 EXPORTS = ("sss_codes_bytes", "sss_status_string", "sss_last_error", "sss_quantize",
-           "sss_dequantize", "sss_gemv", "sss_gemv_multi", "sss_gemm", "sss_workspace_bytes")
+           "sss_dequantize", "sss_gemv", "sss_gemv_multi", "sss_gemm", "sss_workspace_bytes",
+           "sss_gemm_noalloc", "sss_gemm_noalloc_max_scratch_bytes")
 
 GEMV_PDL = 0x1
 GEMV_WEIGHTS_READY = 0x2
@@ -99,6 +100,10 @@ def load(build_if_needed: bool = True):
         L.sss_gemm.restype = i32
         L.sss_workspace_bytes.argtypes = [P, i64, i32]
         L.sss_workspace_bytes.restype = sz
+        L.sss_gemm_noalloc.argtypes = [P, vp, i64, vp, vp, vp]
+        L.sss_gemm_noalloc.restype = i32
+        L.sss_gemm_noalloc_max_scratch_bytes.argtypes = []
+        L.sss_gemm_noalloc_max_scratch_bytes.restype = sz
         _lib = L
         return L
 
@@ -244,3 +249,17 @@ def sss_gemm(qt: QTensor, x, y=None, workspace=None, dev_status=None, stream=Non
                          _ptr(dev_status), _stream(stream))
     _check("sss_gemm", st)
     return y
+
+
+def sss_gemm_noalloc(qt: QTensor, x, y, dev_status=None, stream=None):
+    """sss_gemm with the library's static scratch instead of a workspace;
+    `y` [m, n] fp32 must be given (the call allocates nothing)."""
+    d = qt.desc()
+    st = load().sss_gemm_noalloc(ctypes.byref(d), _ptr(x), x.shape[0], _ptr(y),
+                                 _ptr(dev_status), _stream(stream))
+    _check("sss_gemm_noalloc", st)
+    return y
+
+
+def sss_gemm_noalloc_max_scratch_bytes() -> int:
+    return int(load().sss_gemm_noalloc_max_scratch_bytes())
