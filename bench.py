@@ -530,6 +530,8 @@ def run_micro(args):
     sss.load()
     names = args.matrices.split(",")
     shapes = [inputs.LLAMA3_8B_LAYER[nm] for nm in names]
+    if args.rows:
+        shapes = [(args.rows, kk) for _, kk in shapes]
     k = shapes[0][1]
     G = sss.GRID_ASYM if args.grid == "asym" else (
         sss.GRID_UNSIGNED_SYM if args.grid == "unsigned" else sss.GRID_SIGNED_SYM)
@@ -622,6 +624,7 @@ def main():
     ap.add_argument("--iters", type=int, default=50)
     ap.add_argument("--rotate", type=int, default=8)
     ap.add_argument("--flags", type=int, default=0)
+    ap.add_argument("--rows", type=int, default=0, help="micro: override every matrix's rows")
     args = ap.parse_args()
     if args.micro:
         run_micro(args)

@@ -93,3 +93,20 @@ def test_multi_rejects_mixed_shapes():
     x = torch.zeros(256, dtype=torch.bfloat16, device="cuda")
     with pytest.raises(sss.SssError):
         sss.sss_gemv_multi([a, b], x)
+
+
+@pytest.mark.parametrize("grid", GRIDS)
+@pytest.mark.parametrize("q", QS)
+@pytest.mark.parametrize("k,g", [(1280, 32), (2304, 128), (768, 64)])
+def test_stream_k_not_multiple_of_1024(q, grid, k, g):
+    """k a multiple of 256 only: units of the last stretch of a row."""
+    check_multi([200, 48], k, q, g, grid, 60 + q + k)
+
+
+@pytest.mark.parametrize("g", [32, 64, 128])
+@pytest.mark.parametrize("grid", GRIDS)
+def test_stream_ragged_jobs(g, grid):
+    """Ragged tiles in every job of a fused launch, all group sizes."""
+    check_multi([1000, 33, 7, 250], 3072, 4, g, grid, 70 + g + grid)
+    check_multi([517], 1024, 3, g, grid, 71 + g + grid)
+    check_multi([96, 1], 2048, 2, g, grid, 72 + g + grid)
