@@ -14,9 +14,10 @@
 //    balance the work); a group owns one tile at a time and its warps split
 //    the tile's units (256 codes of every row) round-robin;
 //  * every lane loads the exact bytes it will multiply (its two sub-chunks of
-//    rows g and g+8, and their scales) straight into a ring of registers,
-//    D-1 units ahead of use.  Shared memory holds only the activation
-//    operand.
+//    rows g and g+8, and their scales) straight into a D-slot ring of
+//    registers; a slot is refilled as soon as its unit is multiplied, and
+//    the whole ring is filled before the grid-dependency wait.  Shared
+//    memory holds only the activation operand.
 //  * with KW > 1 a tile's partials meet in a double-buffered shared array
 //    behind mbarriers and only the reducing warp waits; with KW = 1 a warp
 //    owns whole tiles and writes y directly.
@@ -210,7 +211,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   set_tile(0);
   if (!a.early_weights) asm volatile("griddepcontrol.wait;" ::: "memory");
 #pragma unroll
-  for (int d = 0; d < D - 1; ++d)
+  for (int d = 0; d < D; ++d)
     if (d < total) fetch(ring[d]);
   asm volatile("griddepcontrol.wait;" ::: "memory");  // x is produced upstream
 
@@ -224,13 +225,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   // h only when it is the sub-chunk of this quad's own A rows (gq == 2tq + h);
   // otherwise the lane reads zeros
   const bool act0 = gq == 2 * tq, act1 = gq == 2 * tq + 1;
-  const unsigned char* xl = nullptr;  // the lane's B data of the unit being computed
-  const float* bl = nullptr;          // the sums of its two columns' sub-chunks
+  // shared-memory addresses (32-bit) of the lane's B data of the unit being
+  // computed and of the sums of its two columns' sub-chunks
+  const uint32_t xs_a = su32(xs), zero_a = su32(zero), bias_a = su32(bias);
+  uint32_t xl = 0, bl = 0;
   int cleft = 0;
   int64_t ci = 0;
   auto start_tile = [&]() {
-    xl = xs + static_cast<size_t>(kw * 8 + gq) * SL::XPITCH;
-    bl = bias + kw * 8 + 2 * tq;
+    xl = xs_a + static_cast<uint32_t>((kw * 8 + gq) * SL::XPITCH);
+    bl = bias_a + static_cast<uint32_t>((kw * 8 + 2 * tq) * 4);
     cleft = upw;
   };
   start_tile();
@@ -239,23 +242,26 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
     // column 2tq is in dh[0] and 2tq+1 in dh[1]
     float dh[2][4];
 #pragma unroll
-    for (int h = 0; h < 2; ++h) dh[h][0] = dh[h][1] = dh[h][2] = dh[h][3] = 0.f;
-#pragma unroll
     for (int h = 0; h < 2; ++h) {
-      const unsigned char* xp = (h ? act1 : act0) ? xl : zero;
+      const uint32_t xp = (h ? act1 : act0) ? xl : zero_a;
 #pragma unroll
       for (int jm = 0; jm < NP / 2; jm += 2) {
-        const uint4 bv = *reinterpret_cast<const uint4*>(xp + jm * 8);
+        const uint4 bv = lds128(xp + jm * 8);
 #pragma unroll
         for (int jj = 0; jj < 2; ++jj) {
           const int p = 2 * (jm + jj);
-          mma16816(dh[h], unpack_pair<Q>(rg.w[0][h], p), unpack_pair<Q>(rg.w[1][h], p),
-                   unpack_pair<Q>(rg.w[0][h], p + 1), unpack_pair<Q>(rg.w[1][h], p + 1),
-                   jj ? bv.z : bv.x, jj ? bv.w : bv.y);
+          if (jm == 0 && jj == 0)
+            mma16816_z(dh[h], unpack_pair<Q>(rg.w[0][h], p), unpack_pair<Q>(rg.w[1][h], p),
+                       unpack_pair<Q>(rg.w[0][h], p + 1), unpack_pair<Q>(rg.w[1][h], p + 1),
+                       bv.x, bv.y);
+          else
+            mma16816(dh[h], unpack_pair<Q>(rg.w[0][h], p), unpack_pair<Q>(rg.w[1][h], p),
+                     unpack_pair<Q>(rg.w[0][h], p + 1), unpack_pair<Q>(rg.w[1][h], p + 1),
+                     jj ? bv.z : bv.x, jj ? bv.w : bv.y);
         }
       }
     }
-    const float2 bb = *reinterpret_cast<const float2*>(bl);
+    const float2 bb = lds64f(bl);
 #pragma unroll
     for (int hh = 0; hh < 2; ++hh) {
       float s_0, s_1, m_0 = 0.f, m_1 = 0.f;
@@ -279,8 +285,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
         acc[hh] += s_0 * (d0 + bb.x) + s_1 * (d1 + bb.y);
       }
     }
-    xl += static_cast<size_t>(8 * SL::XPITCH) * KW;
-    bl += 8 * KW;
+    xl += static_cast<uint32_t>(8 * SL::XPITCH * KW);
+    bl += static_cast<uint32_t>(32 * KW);
   };
   auto tile_end = [&](int64_t i) {
     const int64_t t = tfirst + i * tstride;
@@ -339,18 +345,32 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   }
   // the units, D at a time so the register ring is indexed at compile time;
   // unit k + D - 1 is loaded while unit k is computed
-  for (int k0 = 0; k0 < total; k0 += D) {
+  auto after_unit = [&]() {
+    if (--cleft == 0) {
+      tile_end(ci);
+      ++ci;
+      start_tile();
+    }
+  };
+  // the units, D at a time so the register ring is indexed at compile time:
+  // unit k is computed from slot k % D, which then takes unit k + D
+  int k0 = 0;
+  for (; k0 + 2 * D <= total; k0 += D) {  // every refill of these D units is in range
+#pragma unroll
+    for (int r = 0; r < D; ++r) {
+      compute(ring[r]);
+      fetch(ring[r]);
+      after_unit();
+    }
+  }
+  for (; k0 < total; k0 += D) {
 #pragma unroll
     for (int r = 0; r < D; ++r) {
       const int k = k0 + r;
       if (k < total) {
-        if (k + D - 1 < total) fetch(ring[(r + D - 1) % D]);
         compute(ring[r]);
-        if (--cleft == 0) {
-          tile_end(ci);
-          ++ci;
-          start_tile();
-        }
+        if (k + D < total) fetch(ring[r]);
+        after_unit();
       }
     }
   }
