@@ -12,18 +12,20 @@
 // 65504).  tcgen05.mma kind::f16 takes both operands in fp16 and accumulates
 // in fp32 in tensor memory.
 //
-// Structure (one CTA per 128-row x BN-token output tile, 6 warps):
+// Structure (one CTA per 128-row x BN-token output tile, 10 warps):
 //   warp 0     TMA producer for the fp16 activation tile (128B swizzle) and
 //              owner of the tensor-memory allocation;
 //   warp 1     a single elected thread issues tcgen05.mma (M=128, N=BN,
 //              K=16 per instruction, 4 per 64-wide k-block) and commits to
 //              the stage's "empty" barrier;
-//   warps 2-5  dequantise: each thread owns one weight row of the tile,
-//              loads that row's codes and scales for the k-block, forms fp16
-//              s*c in natural k order and stores it with the 128B swizzle the
-//              shared-memory descriptor expects; after the last k-block the
-//              same warps drain the fp32 accumulator with tcgen05.ld and store
-//              Y (for a fixed token, a warp writes 32 consecutive floats).
+//   warps 2-9  dequantise: each thread owns one weight row of the tile and
+//              one 32-code half of every 64-wide k-block, loads those codes
+//              and their scale, forms fp16 s*c in natural k order and stores
+//              it with the 128B swizzle the shared-memory descriptor expects;
+//              after the last k-block the same warps drain the fp32
+//              accumulator with tcgen05.ld (each set of four warps one half
+//              of the columns) and store Y (for a fixed token, a warp writes
+//              32 consecutive floats).
 // Every mbarrier wait is bounded (about one second of global time); on
 // expiry the CTA raises SSS_FLAG_TIMEOUT, all roles leave their loops, and
 // the tensor memory is still released.
@@ -39,7 +41,8 @@ namespace {
 
 constexpr int kBM = 128;            // weight rows per tile (MMA M)
 constexpr int kBK = 64;             // k per stage (128 bytes of fp16)
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;      // producer, MMA issuer, 8 dequantising warps
+constexpr int kDqWarps = 8;
 constexpr uint64_t kWaitNs = 1000000000ull;  // bounded waits: 1 s
 
 // ---------------------------------------------------------------------------
@@ -276,7 +279,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
-      mbar_init(&full_a[s], 4);
+      mbar_init(&full_a[s], kDqWarps);
       mbar_init(&full_b[s], 1);
       mbar_init(&empty[s], 1);
     }
@@ -340,28 +343,29 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ---------------- dequantise, then epilogue ----------------
-    const int i = threadIdx.x - 64;  // 0..127: the tile row this thread owns
-    const int64_t r = n0 + i;
+    // thread i owns tile row (i & 127) and, of each 64-wide k-block, the
+    // 32-code half hf = i >> 7
+    const int i = threadIdx.x - 64;  // 0..255
+    const int row_i = i & (kBM - 1);
+    const int hf = i >> 7;
+    const int64_t r = n0 + row_i;
     const bool rok = r < a.n;
     const int64_t nG = a.k / a.G;
     const uint8_t* rowp = a.codes + (rok ? r : 0) * (a.k * Q / 8);
-    const int sw = i & 7;  // swizzle phase of this row
-    // codes and scales of one 64-wide k-block of this row
+    const int sw = row_i & 7;  // swizzle phase of this row
+    // codes and scale (and min) of this thread's half of one k-block
     struct KBlock {
-      uint32_t w[2][4];
-      uint16_t s[2], m[2];
+      uint32_t w[4];
+      uint16_t s, m;
     };
     auto fetch = [&](KBlock& d, int kb) {
       if (kb >= nkb) return;
-#pragma unroll
-      for (int j = 0; j < 2; ++j) {
-        const int64_t kc = static_cast<int64_t>(kb) * kBK + 32 * j;
-        const int64_t grp = kc / a.G;
-        const int sc = static_cast<int>((kc % a.G) / 32);
-        load_sub32<Q>(rowp, grp, sc, a.G, rok, d.w[j]);
-        d.s[j] = rok ? __ldcs(a.scales + r * nG + grp) : static_cast<uint16_t>(0);
-        if constexpr (ASYM) d.m[j] = rok ? __ldcs(a.mins + r * nG + grp) : static_cast<uint16_t>(0);
-      }
+      const int64_t kc = static_cast<int64_t>(kb) * kBK + 32 * hf;
+      const int64_t grp = kc / a.G;
+      const int sc = static_cast<int>((kc % a.G) / 32);
+      load_sub32<Q>(rowp, grp, sc, a.G, rok, d.w);
+      d.s = rok ? __ldcs(a.scales + r * nG + grp) : static_cast<uint16_t>(0);
+      if constexpr (ASYM) d.m = rok ? __ldcs(a.mins + r * nG + grp) : static_cast<uint16_t>(0);
     };
     // the global loads run kPrefetch k-blocks ahead of their use
     constexpr int kPrefetch = 4;
@@ -380,18 +384,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = false;
           break;
         }
-        unsigned char* arow = smem + s * S::STAGE + (i >> 3) * 1024 + sw * 128;
-#pragma unroll
-        for (int j = 0; j < 2; ++j) {  // two 32-code sub-chunks per 64-wide k-block
-          const __half sh = __ushort_as_half(ring[q0].s[j]);
+        unsigned char* arow = smem + s * S::STAGE + (row_i >> 3) * 1024 + sw * 128;
+        {
+          const __half sh = __ushort_as_half(ring[q0].s);
           const __half2 s2 = __halves2half2(sh, sh);
           __half2 m2 = __float2half2_rn(0.f);
           if constexpr (ASYM) {
-            const __half mh = __ushort_as_half(ring[q0].m[j]);
+            const __half mh = __ushort_as_half(ring[q0].m);
             m2 = __halves2half2(mh, mh);
           }
           uint32_t u[16];
-          code_pairs<Q>(ring[q0].w[j], u);
+          code_pairs<Q>(ring[q0].w, u);
           uint32_t out[16];
 #pragma unroll
           for (int p = 0; p < 16; ++p) {
@@ -406,7 +409,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
 #pragma unroll
           for (int cc = 0; cc < 4; ++cc) {  // four 16-byte chunks of 8 elements
-            const int chunk = 4 * j + cc;
+            const int chunk = 4 * hf + cc;
             uint4 v = make_uint4(out[4 * cc], out[4 * cc + 1], out[4 * cc + 2], out[4 * cc + 3]);
             *reinterpret_cast<uint4*>(arow + ((chunk ^ sw) << 4)) = v;
           }
@@ -418,13 +421,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     // ---------------- epilogue ----------------
+    // a warp may read tensor-memory lanes 32*(warp % 4) .. +31; the two sets
+    // of four warps take one half of the columns each
     if (ok && mbar_wait(done, 0, abort)) {
       tc_fence_after();
-      const int sub = warp & 3;  // tensor-memory lane quarter this warp may access
+      const int sub = warp & 3;
       const int row_local = sub * 32 + lane;
       const int64_t rr = n0 + row_local;
+      const int cbeg = (warp < 6) ? 0 : BN / 2;
 #pragma unroll 1
-      for (int c0 = 0; c0 < BN; c0 += 32) {
+      for (int c0 = cbeg; c0 < cbeg + BN / 2; c0 += 32) {
         uint32_t v[32];
         tmem_ld32(tmem + (static_cast<uint32_t>(sub * 32) << 16) + c0, v);
         if (rr < a.n) {
