@@ -12,19 +12,20 @@
 // 65504).  tcgen05.mma kind::f16 takes both operands in fp16 and accumulates
 // in fp32 in tensor memory.
 //
-// Structure (one CTA per 128-row x BN-token output tile, 10 warps):
+// Structure (one CTA per 128-row x BN-token output tile, 18 warps):
 //   warp 0     TMA producer for the fp16 activation tile (128B swizzle) and
 //              owner of the tensor-memory allocation;
 //   warp 1     a single elected thread issues tcgen05.mma (M=128, N=BN,
 //              K=16 per instruction, 4 per 64-wide k-block) and commits to
 //              the stage's "empty" barrier;
-//   warps 2-9  dequantise: each thread owns one weight row of the tile and
-//              one 32-code half of every 64-wide k-block, loads those codes
+//   warps 2-17 dequantise in two sets of eight that fill alternate stages:
+//              each thread owns one weight row of the tile and one 32-code
+//              half of its set's 64-wide k-blocks, loads those codes
 //              and their scale, forms fp16 s*c in natural k order and stores
 //              it with the 128B swizzle the shared-memory descriptor expects;
 //              after the last k-block the same warps drain the fp32
-//              accumulator with tcgen05.ld (each set of four warps one half
-//              of the columns) and store Y (for a fixed token, a warp writes
+//              accumulator with tcgen05.ld (each set of four warps one
+//              quarter of the columns) and store Y (for a fixed token, a warp writes
 //              32 consecutive floats).
 // Every mbarrier wait is bounded (about one second of global time); on
 // expiry the CTA raises SSS_FLAG_TIMEOUT, all roles leave their loops, and
@@ -41,8 +42,9 @@ namespace {
 
 constexpr int kBM = 128;            // weight rows per tile (MMA M)
 constexpr int kBK = 64;             // k per stage (128 bytes of fp16)
-constexpr int kThreads = 320;      // producer, MMA issuer, 8 dequantising warps
-constexpr int kDqWarps = 8;
+constexpr int kDqSets = 2;          // sets of 8 dequantising warps, on alternate k-blocks
+constexpr int kDqWarps = 8;         // warps that fill one stage
+constexpr int kThreads = 64 + 32 * kDqWarps * kDqSets;  // + producer, MMA issuer
 constexpr uint64_t kWaitNs = 1000000000ull;  // bounded waits: 1 s
 
 // ---------------------------------------------------------------------------
@@ -343,11 +345,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ---------------- dequantise, then epilogue ----------------
-    // thread i owns tile row (i & 127) and, of each 64-wide k-block, the
-    // 32-code half hf = i >> 7
-    const int i = threadIdx.x - 64;  // 0..255
+    // thread i owns tile row (i & 127), the 32-code half hf = (i >> 7) & 1 of
+    // each 64-wide k-block, and the k-blocks kb = set, set + kDqSets, ...
+    const int i = threadIdx.x - 64;
     const int row_i = i & (kBM - 1);
-    const int hf = i >> 7;
+    const int hf = (i >> 7) & 1;
+    const int set = i >> 8;
     const int64_t r = n0 + row_i;
     const bool rok = r < a.n;
     const int64_t nG = a.k / a.G;
@@ -367,16 +370,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       d.s = rok ? __ldcs(a.scales + r * nG + grp) : static_cast<uint16_t>(0);
       if constexpr (ASYM) d.m = rok ? __ldcs(a.mins + r * nG + grp) : static_cast<uint16_t>(0);
     };
-    // the global loads run kPrefetch k-blocks ahead of their use
+    // the global loads run kPrefetch of this thread's k-blocks ahead of use
     constexpr int kPrefetch = 4;
     KBlock ring[kPrefetch];
 #pragma unroll
-    for (int q0 = 0; q0 < kPrefetch; ++q0) fetch(ring[q0], q0);
+    for (int q0 = 0; q0 < kPrefetch; ++q0) fetch(ring[q0], set + kDqSets * q0);
     bool ok = true;
-    for (int kb0 = 0; kb0 < nkb && ok; kb0 += kPrefetch) {
+    for (int kb0 = set; kb0 < nkb && ok; kb0 += kDqSets * kPrefetch) {
 #pragma unroll
       for (int q0 = 0; q0 < kPrefetch; ++q0) {
-        const int kb = kb0 + q0;
+        const int kb = kb0 + kDqSets * q0;
         if (kb >= nkb || !ok) break;
         const int s = kb % STAGES;
         const uint32_t ph = static_cast<uint32_t>(kb / STAGES) & 1u;
@@ -417,20 +420,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         fence_proxy_async_smem();  // generic-proxy stores -> visible to the tensor core
         __syncwarp();
         if (lane == 0) mbar_arrive(&full_a[s]);
-        fetch(ring[q0], kb + kPrefetch);
+        fetch(ring[q0], kb + kDqSets * kPrefetch);
       }
     }
     // ---------------- epilogue ----------------
-    // a warp may read tensor-memory lanes 32*(warp % 4) .. +31; the two sets
-    // of four warps take one half of the columns each
+    // a warp may read tensor-memory lanes 32*(warp % 4) .. +31; the four
+    // sets of four warps take one quarter of the columns each
     if (ok && mbar_wait(done, 0, abort)) {
       tc_fence_after();
       const int sub = warp & 3;
       const int row_local = sub * 32 + lane;
       const int64_t rr = n0 + row_local;
-      const int cbeg = (warp < 6) ? 0 : BN / 2;
+      constexpr int kCols = BN / (kDqWarps * kDqSets / 4);
+      const int cbeg = ((warp - 2) >> 2) * kCols;
 #pragma unroll 1
-      for (int c0 = cbeg; c0 < cbeg + BN / 2; c0 += 32) {
+      for (int c0 = cbeg; c0 < cbeg + kCols; c0 += 32) {
         uint32_t v[32];
         tmem_ld32(tmem + (static_cast<uint32_t>(sub * 32) << 16) + c0, v);
         if (rr < a.n) {
