@@ -552,8 +552,8 @@ def run_micro(args):
                       device="cuda") for n, _ in shapes]
     ws = None
     if args.micro == "gemm":
-        ws = torch.empty(max(sss.sss_workspace_bytes(copies[0][0], args.m, sss.OP_GEMM), 16),
-                         dtype=torch.uint8, device="cuda")
+        need = max(sss.sss_workspace_bytes(qt, args.m, sss.OP_GEMM) for qt in copies[0])
+        ws = torch.empty(max(need, 16), dtype=torch.uint8, device="cuda")
 
     def op(c):
         mats = copies[c % args.rotate]

@@ -1,8 +1,8 @@
 // gemv_common.cuh -- pieces of the batch-1 streaming GEMV (gemv_stream.cu):
-// bounded mbarrier waits, the fp16-subnormal
-// code unpack feeding mma.sync m16n8k16, and the staging of the activation
-// vector in mma order with the per-sub-chunk sums of the Appendix B.3
-// row-sum term.
+// bounded mbarrier waits, the fp16-subnormal code unpack feeding
+// mma.sync m16n8k16, and the staging of
+// the activation vector in mma order with the per-sub-chunk sums of the
+// Appendix B.3 row-sum term.
 #pragma once
 
 #include <stdint.h>
@@ -14,21 +14,12 @@ namespace gv {
 
 constexpr uint64_t kWaitNs = 1000000000ull;
 
-template <int Q>
-struct SQ;
-template <>
-struct SQ<4> {
-  // pairs per sub-chunk; 32-bit code words per (row, sub-chunk)
-  static constexpr int NP = 16, NW = 4;
-};
-template <>
-struct SQ<2> {
-  static constexpr int NP = 16, NW = 2;
-};
-template <>
-struct SQ<3> {
-  static constexpr int NP = 32, NW = 3;
-};
+// fp16 pairs per 32-code sub-chunk: every width uses 16 (q=3 merges its two
+// bit planes into 3-bit fields before the mma)
+constexpr int NP = 16;
+// bytes of one sub-chunk's staged activations (16 pairs; no padding: the
+// 16-byte chunks are XOR-swizzled instead, see stage_x)
+constexpr int XPITCH = NP * 4;
 
 __device__ __forceinline__ uint32_t su32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -44,23 +35,18 @@ __device__ __forceinline__ void bar_init(uint64_t* b, uint32_t c) {
 __device__ __forceinline__ void bar_arrive(uint64_t* b) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(b)) : "memory");
 }
-__device__ __forceinline__ void bar_expect(uint64_t* b, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(b)),
-               "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ bool bar_try(uint64_t* b, uint32_t parity) {
+__device__ __forceinline__ bool bar_try(uint32_t b, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
       " selp.u32 %0, 1, 0, p;\n}\n"
       : "=r"(ok)
-      : "r"(su32(b)), "r"(parity)
+      : "r"(b), "r"(parity)
       : "memory");
   return ok != 0;
 }
 // bounded wait; false if it gave up (own limit, or *abort raised elsewhere)
-__device__ __forceinline__ bool bar_wait(uint64_t* b, uint32_t parity, volatile int* abort) {
+__device__ __forceinline__ bool bar_wait_a(uint32_t b, uint32_t parity, volatile int* abort) {
   if (bar_try(b, parity)) return true;
   const uint64_t t0 = gtime();
   for (uint32_t it = 1;; ++it) {
@@ -74,6 +60,10 @@ __device__ __forceinline__ bool bar_wait(uint64_t* b, uint32_t parity, volatile 
     }
   }
 }
+__device__ __forceinline__ bool bar_wait(uint64_t* b, uint32_t parity, volatile int* abort) {
+  return bar_wait_a(su32(b), parity, abort);
+}
+
 __device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
                                          uint32_t a3, uint32_t b0, uint32_t b1) {
   asm volatile(
@@ -106,7 +96,13 @@ __device__ __forceinline__ float2 lds64f(uint32_t addr) {
   return v;
 }
 
-// activation pair p of a 32-code sub-chunk: (element a, element b, multiplier)
+// Activation pair p (0..15) of a 32-code sub-chunk: its two elements and
+// the multiplier that undoes the power of two the code's bit position
+// carries in the fp16 subnormal.
+//   q=4: p = 4w + i covers elements 8w+i and 8w+i+4 (nibble i&1 of a byte
+//        pair, so odd i sits 4 bits up: multiplier 1/16);
+//   q=2 and q=3: p = 8w + e covers elements 16w+e and 16w+e+8, whose 2-bit
+//        fields land at bit 2(e mod 3) after the unpack's shift.
 template <int Q>
 __device__ __forceinline__ void pair_desc(int p, int& ea, int& eb, float& mult) {
   if (Q == 4) {
@@ -114,91 +110,105 @@ __device__ __forceinline__ void pair_desc(int p, int& ea, int& eb, float& mult) 
     ea = 8 * w + i;
     eb = ea + 4;
     mult = (i & 1) ? 0.0625f : 1.f;
-  } else if (Q == 2 || p < 16) {
+  } else {
     const int w = p >> 3, e = p & 7;
     ea = 16 * w + e;
     eb = ea + 8;
     const int m3 = e % 3;
     mult = (m3 == 0) ? 1.f : (m3 == 1 ? 0.25f : 0.0625f);
-  } else {
-    const int j = p - 16;
-    ea = j;
-    eb = j + 16;
-    mult = 4.f / static_cast<float>(1 << (j & 3));
   }
 }
 
-// pair p of a sub-chunk's words as an fp16x2 subnormal operand
+// Pair p of one sub-chunk's code words as an fp16x2 subnormal operand.
+//   q=4: w[0..3] hold the 32 nibbles;
+//   q=2: w[0..1] hold the 32 2-bit codes;
+//   q=3: w[0..1] hold the low 2-bit plane, w[2] the high bit of all 32
+//        codes; the high bit is moved two places above its low field, so
+//        the operand is the 3-bit code at the same bit position.
 template <int Q>
 __device__ __forceinline__ uint32_t unpack_pair(const uint32_t* w, int p) {
   if constexpr (Q == 4) {
     const uint32_t v = (p & 2) ? (w[p >> 2] >> 8) : w[p >> 2];
     return v & ((p & 1) ? 0x00F000F0u : 0x000F000Fu);
   } else {
-    if (Q == 2 || p < 16) {
-      const int e = p & 7;
-      const uint32_t word = w[(p >> 3) & 1];
-      const uint32_t v = e < 3 ? word : (e < 6 ? (word >> 6) : (word >> 12));
-      return v & (0x00030003u << (2 * (e % 3)));
+    const int e = p & 7, pos = 2 * (e % 3);
+    const uint32_t word = w[(p >> 3) & 1];
+    const uint32_t v = e < 3 ? word : (e < 6 ? (word >> 6) : (word >> 12));
+    const uint32_t lo = v & (0x00030003u << pos);
+    if constexpr (Q == 2) {
+      return lo;
     } else {
-      const int j = p - 16;
-      return (w[2] >> (4 * (j >> 2))) & (0x00010001u << (j & 3));
+      // high bits of elements 16w+e and 16w+e+8 at bits e and 16+e
+      const uint32_t hw = __byte_perm(w[2], 0u, (p >> 3) ? 0x4342u : 0x4140u);
+      const int d = pos + 2 - e;
+      const uint32_t hs = d >= 0 ? (hw << d) : (hw >> (-d));
+      return lo | (hs & (0x00040004u << pos));
     }
   }
 }
 
-// Bytes of one 32-code sub-chunk's activations in shared memory, arranged
-// as the mma B operand (NP fp16 pairs) plus 16 bytes of padding that spread
-// the eight columns' rows over the banks.
-template <int Q>
-struct XLayout {
-  static constexpr int XPITCH = SQ<Q>::NP * 4 + 16;
-};
-
 // Stage the bf16 activations x[0..32*nsc) in shared memory for the mma B
-// operand: sub-chunk i (32 elements) becomes NP fp16 pairs in unpack order,
-// each pre-divided by the power of two its code position carries, at
-// xs + i*XPITCH; bias[i] = its sum times 2^-24 (min-max grid) or times
-// -2^(q-1) * 2^-24 (symmetric grids).  Threads tid = 0..nthreads-1 share the
+// operand.  Sub-chunk i (32 elements) becomes NP fp16 pairs in unpack order,
+// each pre-divided by the power of two its code position carries; its four
+// 16-byte chunks c sit at xs + i*XPITCH + 16*(c ^ ((i >> 1) & 3)), a swizzle
+// under which the four sub-chunks one mma reads fall in distinct banks.
+// bias[i] = the sub-chunk's sum times 2^-24 (min-max grid) or times
+// -2^(q-1) * 2^-24 (symmetric grids).  Two threads share a sub-chunk (16
+// elements each); threads tid = 0..nthreads-1 (nthreads even) share the
 // work; the caller synchronises afterwards.
 template <int Q, bool ASYM>
-__device__ __forceinline__ void stage_x(const uint16_t* x, int nsc, unsigned char* xs, float* bias,
+__device__ __forceinline__ void stage_x(const uint16_t* x, int nsc, uint32_t xs_a, float* bias,
                                         int tid, int nthreads) {
-  using SL = XLayout<Q>;
-  constexpr int NP = SQ<Q>::NP;
   constexpr int HALF = 1 << (Q - 1);
-  for (int i = tid; i < nsc; i += nthreads) {
-    const uint4* src = reinterpret_cast<const uint4*>(x + static_cast<int64_t>(i) * 32);
-    uint4 v[4];
+  const int rounds = (2 * nsc + nthreads - 1) / nthreads;
+  for (int r = 0; r < rounds; ++r) {
+    const int t = tid + r * nthreads;
+    const bool valid = t < 2 * nsc;
+    const int i = t >> 1, hf = t & 1;
+    float xv[16];
+    if (valid) {
+      const uint4* src = reinterpret_cast<const uint4*>(x + static_cast<int64_t>(i) * 32 + 16 * hf);
 #pragma unroll
-    for (int c = 0; c < 4; ++c) v[c] = __ldg(src + c);
-    float xv[32];
+      for (int c = 0; c < 2; ++c) {
+        const uint4 v = __ldg(src + c);
+        const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const uint32_t wv[4] = {v[c].x, v[c].y, v[c].z, v[c].w};
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        xv[8 * c + 2 * e] = __uint_as_float(wv[e] << 16);
-        xv[8 * c + 2 * e + 1] = __uint_as_float(wv[e] & 0xFFFF0000u);
+        for (int e = 0; e < 4; ++e) {
+          xv[8 * c + 2 * e] = __uint_as_float(wv[e] << 16);
+          xv[8 * c + 2 * e + 1] = __uint_as_float(wv[e] & 0xFFFF0000u);
+        }
       }
+    } else {
+#pragma unroll
+      for (int e = 0; e < 16; ++e) xv[e] = 0.f;
     }
     float sum = 0.f;
 #pragma unroll
-    for (int e = 0; e < 32; ++e) sum += xv[e];
-    uint32_t pr[NP];
+    for (int e = 0; e < 16; ++e) sum += xv[e];
+    sum += __shfl_xor_sync(0xffffffffu, sum, 1);
+    if (valid) {
+      uint32_t pr[8];
 #pragma unroll
-    for (int p = 0; p < NP; ++p) {
-      int ea, eb;
-      float mult;
-      pair_desc<Q>(p, ea, eb, mult);
-      __half2 hv = __floats2half2_rn(xv[ea] * mult, xv[eb] * mult);
-      pr[p] = *reinterpret_cast<uint32_t*>(&hv);
+      for (int j = 0; j < 8; ++j) {
+        // pair 8hf + j; both its elements lie in this half, at the same
+        // offsets from the half's start for either half
+        int ea, eb;
+        float mult;
+        pair_desc<Q>(j, ea, eb, mult);
+        __half2 hv = __floats2half2_rn(xv[ea] * mult, xv[eb] * mult);
+        pr[j] = *reinterpret_cast<uint32_t*>(&hv);
+      }
+      const uint32_t row = xs_a + static_cast<uint32_t>(i * XPITCH);
+      const int sw = (i >> 1) & 3;
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        const uint32_t dst = row + 16u * static_cast<uint32_t>((2 * hf + c) ^ sw);
+        asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(dst), "r"(pr[4 * c]),
+                     "r"(pr[4 * c + 1]), "r"(pr[4 * c + 2]), "r"(pr[4 * c + 3])
+                     : "memory");
+      }
+      if (hf == 0) bias[i] = ASYM ? sum * 0x1p-24f : -static_cast<float>(HALF) * 0x1p-24f * sum;
     }
-    unsigned char* dst = xs + static_cast<size_t>(i) * SL::XPITCH;
-#pragma unroll
-    for (int c = 0; c < NP / 4; ++c)
-      *reinterpret_cast<uint4*>(dst + 16 * c) = make_uint4(pr[4 * c], pr[4 * c + 1], pr[4 * c + 2], pr[4 * c + 3]);
-    bias[i] = ASYM ? sum * 0x1p-24f : -static_cast<float>(HALF) * 0x1p-24f * sum;
   }
 }
 

@@ -67,10 +67,6 @@ struct StreamArgs {
 
 template <int Q, bool ASYM, int G, int D>
 __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_constant__ StreamArgs a) {
-  using SL = XLayout<Q>;
-  constexpr int NP = SQ<Q>::NP;
-  constexpr int HALF = 1 << (Q - 1);
-  constexpr int LGG = G == 32 ? 5 : (G == 64 ? 6 : 7);
   constexpr int R = 16;
   extern __shared__ __align__(128) unsigned char smem[];
 
@@ -84,9 +80,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
 
   // ---- shared memory carve-up ----
   unsigned char* xs = smem;                                                 // [nsc][XPITCH]
-  float* bias = reinterpret_cast<float*>(xs + static_cast<size_t>(nsc) * SL::XPITCH);  // [nsc]
-  unsigned char* zero = reinterpret_cast<unsigned char*>(bias + nsc);      // 128 B
-  uint64_t* pready = reinterpret_cast<uint64_t*>(zero + 128);              // [kWarps][2]
+  float* bias = reinterpret_cast<float*>(xs + static_cast<size_t>(nsc) * XPITCH);  // [nsc]
+  uint64_t* pready = reinterpret_cast<uint64_t*>(bias + ((nsc + 1) & ~1));  // [kWarps][2]
   uint64_t* pfree = pready + 2 * kWarps;                                   // [kWarps][2]
   float* part = reinterpret_cast<float*>(pfree + 2 * kWarps);              // [kWarps][2][R]
   volatile int* abort = reinterpret_cast<volatile int*>(part + 2 * kWarps * R);
@@ -105,7 +100,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
     *abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  for (int i = threadIdx.x; i < 32; i += blockDim.x) reinterpret_cast<uint32_t*>(zero)[i] = 0u;
   // allow the next kernel in the stream to be scheduled as SMs free up
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
@@ -129,7 +123,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   // the lane's byte offset in a unit's codes (sub-chunks 2tq, 2tq+1; q=3
   // addresses its planes per sub-chunk below) and its scale index in the
   // unit: the pair of groups 2tq, 2tq+1 for g=32, else its one group
-  const int lane_c = Q == 4 ? 32 * tq : (Q == 2 ? 16 * tq : 0);
+  // q=3: the lane's two sub-chunks are 24 contiguous bytes at 24tq (g=32:
+  // two groups [lo hi | lo hi]; g=64: one group [lo lo | hi hi]), or for
+  // g=128 16 low-plane bytes at 48(tq>>1) + 16(tq&1) and 8 high-plane bytes
+  // 32 bytes further on
+  const int lane_c = Q == 4 ? 32 * tq : (Q == 2 ? 16 * tq : (G == 128 ? 48 * (tq >> 1) + 16 * (tq & 1) : 24 * tq));
   const int lane_s = G == 32 ? 2 * tq : (G == 64 ? tq : (tq >> 1));
 
   // the code/scale/min pointers of rows g and g+8 of this warp's i-th tile,
@@ -181,16 +179,21 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
         const uint4 v = __ldcs(reinterpret_cast<const uint4*>(rp));
         rg.w[hh][0][0] = v.x; rg.w[hh][0][1] = v.y;
         rg.w[hh][1][0] = v.z; rg.w[hh][1][1] = v.w;
-      } else {  // q=3: two low-plane words and one high-plane word per sub-chunk
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int e0 = (2 * tq + h) * 32;  // within the unit (units hold whole groups)
-          const int gbyte = (e0 >> LGG) * (3 * G / 8);
-          const int sc = (e0 & (G - 1)) >> 5;
-          const uint32_t* lo = reinterpret_cast<const uint32_t*>(rp + gbyte + 8 * sc);
-          rg.w[hh][h][0] = __ldcs(lo);
-          rg.w[hh][h][1] = __ldcs(lo + 1);
-          rg.w[hh][h][2] = __ldcs(reinterpret_cast<const uint32_t*>(rp + gbyte + G / 4 + 4 * sc));
+      } else if constexpr (G == 128) {  // q=3: [lo lo] (16 B) and [hi hi] (8 B)
+        const uint4 lo = __ldcs(reinterpret_cast<const uint4*>(rp));
+        const uint2 hi = __ldcs(reinterpret_cast<const uint2*>(rp + 32 - 8 * (tq & 1)));
+        rg.w[hh][0][0] = lo.x; rg.w[hh][0][1] = lo.y; rg.w[hh][0][2] = hi.x;
+        rg.w[hh][1][0] = lo.z; rg.w[hh][1][1] = lo.w; rg.w[hh][1][2] = hi.y;
+      } else {  // q=3, g=32 / 64: 24 contiguous bytes
+        const uint2 p0 = __ldcs(reinterpret_cast<const uint2*>(rp));
+        const uint2 p1 = __ldcs(reinterpret_cast<const uint2*>(rp + 8));
+        const uint2 p2 = __ldcs(reinterpret_cast<const uint2*>(rp + 16));
+        if constexpr (G == 32) {
+          rg.w[hh][0][0] = p0.x; rg.w[hh][0][1] = p0.y; rg.w[hh][0][2] = p1.x;
+          rg.w[hh][1][0] = p1.y; rg.w[hh][1][1] = p2.x; rg.w[hh][1][2] = p2.y;
+        } else {
+          rg.w[hh][0][0] = p0.x; rg.w[hh][0][1] = p0.y; rg.w[hh][0][2] = p2.x;
+          rg.w[hh][1][0] = p1.x; rg.w[hh][1][1] = p1.y; rg.w[hh][1][2] = p2.y;
         }
       }
       if constexpr (G == 32) {
@@ -216,7 +219,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   asm volatile("griddepcontrol.wait;" ::: "memory");  // x is produced upstream
 
   // ---- stage the activations in mma order, and per-sub-chunk sums ----
-  stage_x<Q, ASYM>(a.x, nsc, xs, bias, threadIdx.x, kThreads);
+  stage_x<Q, ASYM>(a.x, nsc, su32(xs), bias, threadIdx.x, kThreads);
   __syncthreads();
 
   bool ok = true;
@@ -225,14 +228,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   // h only when it is the sub-chunk of this quad's own A rows (gq == 2tq + h);
   // otherwise the lane reads zeros
   const bool act0 = gq == 2 * tq, act1 = gq == 2 * tq + 1;
+  // swizzle of the staged activations of sub-chunk 8u + gq
+  const int xsw = (gq >> 1) & 3;
   // shared-memory addresses (32-bit) of the lane's B data of the unit being
   // computed and of the sums of its two columns' sub-chunks
-  const uint32_t xs_a = su32(xs), zero_a = su32(zero), bias_a = su32(bias);
+  const uint32_t xs_a = su32(xs), bias_a = su32(bias);
   uint32_t xl = 0, bl = 0;
   int cleft = 0;
   int64_t ci = 0;
   auto start_tile = [&]() {
-    xl = xs_a + static_cast<uint32_t>((kw * 8 + gq) * SL::XPITCH);
+    xl = xs_a + static_cast<uint32_t>((kw * 8 + gq) * XPITCH);
     bl = bias_a + static_cast<uint32_t>((kw * 8 + 2 * tq) * 4);
     cleft = upw;
   };
@@ -243,10 +248,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
     float dh[2][4];
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      const uint32_t xp = (h ? act1 : act0) ? xl : zero_a;
+      const bool act = h ? act1 : act0;
 #pragma unroll
       for (int jm = 0; jm < NP / 2; jm += 2) {
-        const uint4 bv = lds128(xp + jm * 8);
+        uint4 bv = make_uint4(0u, 0u, 0u, 0u);
+        if (act) bv = lds128(xl + 16u * static_cast<uint32_t>((jm >> 1) ^ xsw));
 #pragma unroll
         for (int jj = 0; jj < 2; ++jj) {
           const int p = 2 * (jm + jj);
@@ -285,7 +291,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
         acc[hh] += s_0 * (d0 + bb.x) + s_1 * (d1 + bb.y);
       }
     }
-    xl += static_cast<uint32_t>(8 * SL::XPITCH * KW);
+    xl += static_cast<uint32_t>(8 * XPITCH * KW);
     bl += static_cast<uint32_t>(32 * KW);
   };
   auto tile_end = [&](int64_t i) {
@@ -379,12 +385,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
 
 template <int Q, bool ASYM>
 size_t smem_bytes(int64_t k, int depth) {
-  using SL = XLayout<Q>;
   const int64_t nsc = k / 32;
-  // activations | sums | zeros | 4*kWarps barriers | partials | flag
+  // activations | sums | 4*kWarps barriers | partials | flag
   (void)depth;
-  return static_cast<size_t>(nsc) * SL::XPITCH +
-         4 * nsc + 128 + 8 * 4 * kWarps + 4 * 2 * kWarps * 16 + 16;
+  return static_cast<size_t>(nsc) * XPITCH + 4 * ((nsc + 1) & ~int64_t{1}) +
+         8 * 4 * kWarps + 4 * 2 * kWarps * 16 + 16;
 }
 
 template <int Q, bool ASYM, int G, int D>
@@ -431,7 +436,7 @@ cudaError_t launch_q(const sss_qtensor_t* const* ts, StreamArgs& a, bool pdl,
   const int64_t per_cta = (tiles + grid - 1) / grid;
   int best = 0;
   int64_t best_cost = INT64_MAX;
-  for (int lg = 0; lg <= 4; ++lg) {
+  for (int lg = 0; (1 << lg) <= kWarps; ++lg) {
     const int kwn = 1 << lg;
     if (kwn > 1 && kwn > nunits) break;
     const int64_t ngrp = kWarps >> lg;
@@ -462,7 +467,7 @@ bool gemv_stream_eligible(const sss_qtensor_t& t, const uint16_t* x) {
   if (t.grid == SSS_GRID_ASYM && !al(t.mins, 4)) return false;
   // the staged activations must fit in shared memory
   const int64_t nsc = t.k / 32;
-  const int64_t xbytes = nsc * ((t.q == 3 ? 32 : 16) * 4 + 16 + 4);
+  const int64_t xbytes = nsc * (gv::XPITCH + 4);
   return xbytes + 4096 <= 227 * 1024;
 }
 
