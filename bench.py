@@ -604,6 +604,143 @@ def run_micro(args):
                       "iters": args.iters, "rotate": args.rotate}), flush=True)
 
 
+def _graph_time_us(fn, iters: int) -> float:
+    """Mean µs per call of fn(i), i = 0..iters-1, captured in one CUDA graph
+    and replayed once after a warm replay."""
+    import torch
+
+    for i in range(3):
+        fn(i)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    cs = torch.cuda.Stream()
+    with torch.cuda.graph(graph, stream=cs):
+        for i in range(iters):
+            fn(i)
+    graph.replay()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    graph.replay()
+    b.record()
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) * 1e3 / iters
+
+
+def sweep_qwen3_quantize(args):
+    """Weight quantization of a whole Qwen3-32B-shaped model (64 layers of
+    q/k/v/o/gate/up/down, 31.2G weights), signed grid, q in {2, 3} x group
+    in {32, 128}.  Each layer's fp32 weights are generated on the device into
+    reused buffers (heavy-tailed, with outlier channels); every quantize
+    launch is timed with CUDA events and the rate is weights over the sum of
+    kernel times.  Prints one JSON line per (q, group) and a summary."""
+    import torch
+
+    from paper_2607_08779_gb300 import inputs, sss
+
+    torch.cuda.set_device(0)
+    sss.load()
+    hbm, _, _, peak_kind = peaks()
+    shapes = list(inputs.QWEN3_32B_LAYER.items())
+    layers = args.layers if args.layers != 32 else inputs.QWEN3_32B_LAYERS
+    variants = [(q, g) for q in (2, 3) for g in (32, 128)]
+    G = sss.GRID_SIGNED_SYM
+    w = [torch.empty((n, k), dtype=torch.float32, device="cuda") for _, (n, k) in shapes]
+    outs = {v: [sss.empty_qtensor(n, k, v[0], v[1], G) for _, (n, k) in shapes] for v in variants}
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ms = {v: 0.0 for v in variants}
+    weights = 0
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2 * len(variants))]
+    for layer in range(layers):
+        for mi, (_, (n, k)) in enumerate(shapes):
+            inputs.student_t_weights_cuda(n, k, inputs.weight_seed(4, layer, mi), out=w[mi])
+        weights += sum(n * k for _, (n, k) in shapes)
+        for vi, v in enumerate(variants):
+            ev[2 * vi].record()
+            for mi in range(len(shapes)):
+                sss.sss_quantize(w[mi], v[0], v[1], G, out=outs[v][mi], dev_status=status)
+            ev[2 * vi + 1].record()
+        torch.cuda.synchronize()
+        for vi, v in enumerate(variants):
+            ms[v] += ev[2 * vi].elapsed_time(ev[2 * vi + 1])
+    summary = []
+    for v in variants:
+        q, g = v
+        bpw = 4 + q / 8 + 2 / g
+        gw = weights / (ms[v] * 1e-3) / 1e9
+        line = {"sweep": "qwen3_32b_quantize", "layers": layers, "q": q, "group": g,
+                "grid": "signed", "weights": weights, "kernel_ms": round(ms[v], 3),
+                "gweights_per_s": round(gw, 1), "gbs": round(gw * bpw, 1),
+                "frac_hbm": round(gw * bpw / hbm, 4), "peak_source": peak_kind,
+                "device_status": int(status.item())}
+        summary.append(line)
+        print(json.dumps(line), flush=True)
+    return summary
+
+
+def sweep_grids(args):
+    """The grid comparison on the 4096x4096 shape (heavy-tailed weights with
+    outlier channels): unsigned symmetric vs signed symmetric vs min-max, at
+    q in {2, 3, 4} and group 32 / 128.  Per format: the per-group l2 error of
+    the stored (fp16-scale) dequantised weights (mean, p50, p99, fp64), the
+    fraction of groups with |C_gamma| <= |C_-gamma| (symmetric grids), and
+    the decode GEMV GB/s at batch 1 / 4 / 16, timed in a CUDA graph over more
+    copies of the packed matrix than L2 holds."""
+    import torch
+
+    from paper_2607_08779_gb300 import inputs, sss
+
+    torch.cuda.set_device(0)
+    sss.load()
+    hbm, _, _, peak_kind = peaks()
+    n = k = 4096
+    l2 = torch.cuda.get_device_properties(0).L2_cache_size
+    W = inputs.student_t_weights_cuda(n, k, inputs.weight_seed(5, 0, 0))
+    Wd = W.double()
+    xs = {b: inputs.normal_bf16_cuda((b, k), 50 + b) for b in (1, 4, 16)}
+    rows = []
+    for gname, grid in (("unsigned", sss.GRID_UNSIGNED_SYM), ("signed", sss.GRID_SIGNED_SYM),
+                        ("asym", sss.GRID_ASYM)):
+        for q in (2, 3, 4):
+            for g in (32, 128):
+                cc = torch.zeros((n, k // g, 2), dtype=torch.uint8, device="cuda")
+                st = torch.zeros(1, dtype=torch.int32, device="cuda")
+                qt = sss.sss_quantize(W, q, g, grid, clip_counts=cc, dev_status=st)
+                what = sss.sss_dequantize(qt)
+                err = (Wd - what.double()).view(n, k // g, g).pow(2).sum(-1).sqrt().flatten()
+                qs = torch.quantile(err.float(), torch.tensor([0.5, 0.99], device="cuda"))
+                line = {"sweep": "grids", "grid": gname, "q": q, "group": g,
+                        "l2_err_mean": float(err.mean()), "l2_err_p50": float(qs[0]),
+                        "l2_err_p99": float(qs[1]),
+                        "frac_groups_clip_self_le_other": (
+                            None if grid == sss.GRID_ASYM else
+                            float((cc[..., 0] <= cc[..., 1]).float().mean())),
+                        "device_status": int(st.item())}
+                packed = qt.codes.numel() + qt.scales.numel() * 2 + (
+                    qt.mins.numel() * 2 if qt.mins is not None else 0)
+                copies = max(4, -(-4 * l2 // packed))
+                pool = [qt] + [sss.QTensor(qt.n, qt.k, q, g, grid, qt.codes.clone(),
+                                           qt.scales.clone(),
+                                           None if qt.mins is None else qt.mins.clone())
+                               for _ in range(copies - 1)]
+                for b, x in xs.items():
+                    y = torch.empty((b, n), dtype=torch.float32, device="cuda")
+                    need = sss.sss_workspace_bytes(qt, b, sss.OP_GEMV)
+                    ws = torch.empty(max(need, 16), dtype=torch.uint8, device="cuda")
+                    us = _graph_time_us(
+                        lambda i: sss.sss_gemv(pool[i % copies], x, y=y, workspace=ws),
+                        max(args.iters, 2 * copies))
+                    nbytes = packed + 2 * b * k + 4 * b * n
+                    line["gemv_b%d_us" % b] = round(us, 3)
+                    line["gemv_b%d_gbs" % b] = round(nbytes / us / 1e3, 1)
+                line["gemv_b1_frac_hbm"] = round(line["gemv_b1_gbs"] / hbm, 4)
+                line["peak_source"] = peak_kind
+                rows.append(line)
+                print(json.dumps(line), flush=True)
+                del pool
+    return rows
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -625,7 +762,16 @@ def main():
     ap.add_argument("--rotate", type=int, default=8)
     ap.add_argument("--flags", type=int, default=0)
     ap.add_argument("--rows", type=int, default=0, help="micro: override every matrix's rows")
+    ap.add_argument("--sweep", choices=["qwen3_quantize", "grids"],
+                    help="measurement sweeps: whole-model quantization of Qwen3-32B shapes, "
+                         "or the unsigned / signed / min-max grid comparison")
     args = ap.parse_args()
+    if args.sweep == "qwen3_quantize":
+        sweep_qwen3_quantize(args)
+        return
+    if args.sweep == "grids":
+        sweep_grids(args)
+        return
     if args.micro:
         run_micro(args)
         return
