@@ -547,9 +547,9 @@ def run_micro(args):
                 mats.append(sss.sss_quantize(w, q, g, G))
                 del w
         copies.append(mats)
-    x = inputs.normal_bf16_cuda((args.m if args.micro == "gemm" else 1, k), 5)
-    ys = [torch.empty((args.m if args.micro == "gemm" else 1, n), dtype=torch.float32,
-                      device="cuda") for n, _ in shapes]
+    rows_x = args.m if args.micro == "gemm" else (args.batch if args.micro == "gemv_single" else 1)
+    x = inputs.normal_bf16_cuda((rows_x, k), 5)
+    ys = [torch.empty((rows_x, n), dtype=torch.float32, device="cuda") for n, _ in shapes]
     ws = None
     if args.micro == "gemm":
         need = max(sss.sss_workspace_bytes(qt, args.m, sss.OP_GEMM) for qt in copies[0])
@@ -594,11 +594,11 @@ def run_micro(args):
         elif args.micro == "gemm":
             nbytes += packed + 2 * args.m * kk + 4 * args.m * n
         else:
-            nbytes += packed + 4 * n
-    if args.micro != "quantize":
-        nbytes += 2 * k * (args.m if args.micro == "gemm" else 1)
-    flops = 2 * (args.m if args.micro == "gemm" else 1) * sum(n * kk for n, kk in shapes)
-    print(json.dumps({"micro": args.micro, "matrices": names, "q": q, "group": g,
+            nbytes += packed + 4 * n * rows_x
+    if args.micro not in ("quantize", "gemm"):
+        nbytes += 2 * k * rows_x
+    flops = 2 * rows_x * sum(n * kk for n, kk in shapes)
+    print(json.dumps({"micro": args.micro, "matrices": names, "q": q, "group": g, "rows_x": rows_x,
                       "grid": args.grid, "us_per_call": round(us, 3),
                       "gbs": round(nbytes / us / 1e3, 1), "tflops": round(flops / us / 1e6, 2),
                       "iters": args.iters, "rotate": args.rotate}), flush=True)
@@ -758,6 +758,7 @@ def main():
     ap.add_argument("--group", type=int, default=32)
     ap.add_argument("--grid", choices=["signed", "unsigned", "asym"], default="signed")
     ap.add_argument("--m", type=int, default=512)
+    ap.add_argument("--batch", type=int, default=1, help="micro gemv_single: activation rows")
     ap.add_argument("--iters", type=int, default=50)
     ap.add_argument("--rotate", type=int, default=8)
     ap.add_argument("--flags", type=int, default=0)

@@ -139,7 +139,12 @@ sss_status_t sss_dequantize(const sss_qtensor_t* qt, void* out,
  * sss_gemv -- decode GEMV y[b][r] = sum_k w^[r][k] * x[b][k] with the
  * dequantisation fused (Appendix B.3: y = sum_b s * (integer dot) for the
  * symmetric formats, plus the row-sum term sum_b m * sum_{k in b} x for
- * ASYM).  fp32 accumulation; deterministic (no atomics).
+ * ASYM).  fp32 accumulation; deterministic (no atomics).  At batch 1 the
+ * integer codes meet the activations exactly and the group scale is applied
+ * in fp32.  At batch 2..16 (k a multiple of 256), the batch fills the
+ * tensor-core columns, so each weight enters the product as w^ rounded once
+ * to fp16 (<= 2^-11 relative, as in sss_gemm); that operand overflows if
+ * |w^| * 16 >= 65504.
  *   qt        [in]  packed tensor; codes 16-byte aligned, scales/mins 4-byte
  *                   aligned.
  *   x_bf16    [in]  device bf16 [batch][k], 16-byte aligned.
@@ -148,7 +153,7 @@ sss_status_t sss_dequantize(const sss_qtensor_t* qt, void* out,
  *   workspace [in]  device scratch of ws_bytes >= sss_workspace_bytes(qt,
  *                   batch, SSS_OP_GEMV) bytes, 16-byte aligned, or NULL when
  *                   that size is 0.  Its contents on entry are ignored.
- *   dev_status [out] nullable; unused by the GEMV (reserved).
+ *   dev_status [out] nullable; SSS_FLAG_TIMEOUT if a bounded wait expired.
  * Errors: SSS_E_ARG, SSS_E_ALIGN, SSS_E_WORKSPACE, SSS_E_CUDA.
  */
 sss_status_t sss_gemv(const sss_qtensor_t* qt, const uint16_t* x_bf16,

@@ -185,6 +185,10 @@ sss_status_t sss_gemv(const sss_qtensor_t* qt, const uint16_t* x_bf16, int32_t b
     return finish("sss_gemv", launch_gemv_stream(one, yy, 1, x_bf16, 0u, dev_status,
                                                  static_cast<cudaStream_t>(stream)));
   }
+  if (batch >= 2 && gemv_batch_eligible(*qt, x_bf16, batch, y)) {
+    return finish("sss_gemv", launch_gemv_batch(*qt, x_bf16, batch, y, dev_status,
+                                                static_cast<cudaStream_t>(stream)));
+  }
   return finish("sss_gemv", launch_gemv(*qt, x_bf16, batch, y, workspace,
                                         static_cast<cudaStream_t>(stream)));
 }

@@ -39,6 +39,10 @@ cudaError_t launch_gemv_stream(const sss_qtensor_t* const* ts, float* const* ys,
                                const uint16_t* x, uint32_t flags, uint32_t* status,
                                cudaStream_t stream);
 
+bool gemv_batch_eligible(const sss_qtensor_t& t, const uint16_t* x, int batch, const float* y);
+cudaError_t launch_gemv_batch(const sss_qtensor_t& t, const uint16_t* x, int batch, float* y,
+                              uint32_t* status, cudaStream_t stream);
+
 size_t gemm_workspace_bytes(const sss_qtensor_t& t, int64_t m);
 cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m,
                         float* y, void* workspace, uint32_t* status,
