@@ -65,6 +65,22 @@ def test_gemv_batched_q(q, batch):
     run_case(64, 2048, q, 128, sss.GRID_ASYM, batch, 11 + q)
 
 
+@pytest.mark.parametrize("batch", [5, 9, 16])
+@pytest.mark.parametrize("q,grid", [(4, sss.GRID_SIGNED_SYM), (3, sss.GRID_ASYM), (2, sss.GRID_UNSIGNED_SYM)])
+def test_gemv_batched_long_k_slabs(q, grid, batch):
+    # k = 14336 (the down_proj width): at batch > 8 the staged activations
+    # of all 56 units exceed shared memory, so the batched kernel runs the k
+    # range in several slabs and adds each slab's result into y; 100 rows is
+    # not a multiple of the 16-row tile
+    run_case(100, 14336, q, 32, grid, batch, 900 + 10 * q + batch)
+
+
+@pytest.mark.parametrize("batch", [2, 3, 8, 13])
+@pytest.mark.parametrize("g", [32, 64, 128])
+def test_gemv_batched_ragged_rows(g, batch):
+    run_case(75, 2048, 4, g, sss.GRID_SIGNED_SYM, batch, 40 + g + batch)
+
+
 def test_gemv_4096_square_q4_signed():
     """The 4096x4096 q=4 g=32 signed-symmetric case, every output checked."""
     run_case(4096, 4096, 4, 32, sss.GRID_SIGNED_SYM, 1, 1, outliers=False)
