@@ -741,6 +741,71 @@ def sweep_grids(args):
     return rows
 
 
+def sweep_margins(args):
+    """Cardinality margin against realised error gain (Remark
+    rem:cardinality-margin) on every group of one Llama3-8B-shaped layer
+    (heavy-tailed weights with outlier channels), group 32, q in {2, 3, 4}.
+
+    Per group: gamma* is the sign the signed grid stored; the margin is
+    m = |C_-gamma*| - |C_gamma*| from the signed quantizer's clip counts; the
+    gain is g = ||w - Q_-gamma*(w)||^2 - ||w - Q_gamma*(w)||^2, both errors
+    of the stored (fp16-scale) dequantised weights in fp64.  Q_+1 is the
+    unsigned grid on w; Q_-1(w) = -Q_+1(-w), the unsigned grid on -w.
+    Groups with M = 0 are left out."""
+    import torch
+
+    from paper_2607_08779_gb300 import inputs, sss
+
+    torch.cuda.set_device(0)
+    sss.load()
+    g = 32
+    rows = []
+    for q in (2, 3, 4):
+        tot = {"groups": 0, "m_ge0": 0, "m_gt0": 0, "m_gt0_g_gt0": 0, "m_lt0": 0,
+               "m_lt0_g_gt0": 0, "m_eq0": 0, "m_eq0_g_gt0": 0, "g_gt0": 0}
+        for mi, (name, (n, k)) in enumerate(inputs.LLAMA3_8B_LAYER.items()):
+            w = inputs.student_t_weights_cuda(n, k, inputs.weight_seed(2, 0, mi))
+            cc = torch.zeros((n, k // g, 2), dtype=torch.uint8, device="cuda")
+            st = torch.zeros(1, dtype=torch.int32, device="cuda")
+            qs = sss.sss_quantize(w, q, g, sss.GRID_SIGNED_SYM, clip_counts=cc, dev_status=st)
+            qp = sss.sss_quantize(w, q, g, sss.GRID_UNSIGNED_SYM, dev_status=st)
+            qm = sss.sss_quantize(-w, q, g, sss.GRID_UNSIGNED_SYM, dev_status=st)
+            wd = w.double().view(n, k // g, g)
+            e_plus = (wd - sss.sss_dequantize(qp).double().view(n, k // g, g)).pow(2).sum(-1)
+            e_minus = (wd + sss.sss_dequantize(qm).double().view(n, k // g, g)).pow(2).sum(-1)
+            s_bits = qs.scales.view(torch.int16)
+            neg = (s_bits < 0)                    # stored sign bit: gamma* = -1
+            live = (s_bits & 0x7FFF) != 0         # M > 0
+            gain = torch.where(neg, e_plus - e_minus, e_minus - e_plus)
+            m = cc[..., 1].int() - cc[..., 0].int()
+            gp = gain > 0
+            tot["groups"] += int(live.sum())
+            tot["m_ge0"] += int((live & (m >= 0)).sum())
+            tot["m_gt0"] += int((live & (m > 0)).sum())
+            tot["m_gt0_g_gt0"] += int((live & (m > 0) & gp).sum())
+            tot["m_lt0"] += int((live & (m < 0)).sum())
+            tot["m_lt0_g_gt0"] += int((live & (m < 0) & gp).sum())
+            tot["m_eq0"] += int((live & (m == 0)).sum())
+            tot["m_eq0_g_gt0"] += int((live & (m == 0) & gp).sum())
+            tot["g_gt0"] += int((live & gp).sum())
+            if int(st.item()) != 0:
+                tot["device_status"] = int(st.item())
+            del w, wd, e_plus, e_minus, gain
+        n_g = max(1, tot["groups"])
+        line = {"sweep": "margins", "layer": "llama3_8b", "q": q, "group": g,
+                "groups": tot["groups"],
+                "frac_condition_m_ge0": round(tot["m_ge0"] / n_g, 5),
+                "frac_m_gt0": round(tot["m_gt0"] / n_g, 5),
+                "frac_gain_pos_given_m_gt0": round(tot["m_gt0_g_gt0"] / max(1, tot["m_gt0"]), 5),
+                "frac_gain_pos_given_m_eq0": round(tot["m_eq0_g_gt0"] / max(1, tot["m_eq0"]), 5),
+                "frac_gain_pos_given_m_lt0": round(tot["m_lt0_g_gt0"] / max(1, tot["m_lt0"]), 5),
+                "frac_gain_pos": round(tot["g_gt0"] / n_g, 5),
+                "device_status": tot.get("device_status", 0)}
+        rows.append(line)
+        print(json.dumps(line), flush=True)
+    return rows
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -763,7 +828,7 @@ def main():
     ap.add_argument("--rotate", type=int, default=8)
     ap.add_argument("--flags", type=int, default=0)
     ap.add_argument("--rows", type=int, default=0, help="micro: override every matrix's rows")
-    ap.add_argument("--sweep", choices=["qwen3_quantize", "grids"],
+    ap.add_argument("--sweep", choices=["qwen3_quantize", "grids", "margins"],
                     help="measurement sweeps: whole-model quantization of Qwen3-32B shapes, "
                          "or the unsigned / signed / min-max grid comparison")
     args = ap.parse_args()
@@ -772,6 +837,9 @@ def main():
         return
     if args.sweep == "grids":
         sweep_grids(args)
+        return
+    if args.sweep == "margins":
+        sweep_margins(args)
         return
     if args.micro:
         run_micro(args)
