@@ -81,6 +81,15 @@ def test_gemv_batched_ragged_rows(g, batch):
     run_case(75, 2048, 4, g, sss.GRID_SIGNED_SYM, batch, 40 + g + batch)
 
 
+@pytest.mark.parametrize("batch", [1, 16])
+def test_gemv_qwen_down_width(batch):
+    # the widest reduction of the configs (Qwen3-32B down_proj, k = 25600):
+    # 100 units per row for the batch-1 kernel, eight x slabs for the
+    # batched one; 264 rows (a ragged last tile), every output checked
+    k = inputs.QWEN3_32B_LAYER["down_proj"][1]
+    run_case(264, k, 2, 32, sss.GRID_SIGNED_SYM, batch, 4242 + batch)
+
+
 def test_gemv_4096_square_q4_signed():
     """The 4096x4096 q=4 g=32 signed-symmetric case, every output checked."""
     run_case(4096, 4096, 4, 32, sss.GRID_SIGNED_SYM, 1, 1, outliers=False)
