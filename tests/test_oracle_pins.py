@@ -212,6 +212,20 @@ def test_sign_rule_against_both_signs(q):
 
 
 @pytest.mark.parametrize("q", QS)
+def test_negative_sign_is_the_unsigned_grid_on_the_negated_group(q):
+    # Q_-1(w) = -Q_+1(-w): the quantizer with scale -alpha gives the same
+    # codes as the unsigned grid applied to -w (the same exact quotient),
+    # with the opposite scale.  The margin/gain sweep forms Q_-gamma* this
+    # way from the unsigned grid.
+    for w in _groups_for_sign_tests():
+        neg = oracle.quantize_group_gamma(w, q, -1)
+        flip = oracle.quantize_group(-np.asarray(w, np.float32), q, oracle.GRID_UNSIGNED_SYM)
+        assert np.array_equal(neg["c"], flip["c"])
+        assert np.array_equal(neg["c_pre"], flip["c_pre"])
+        assert neg["s32"] == -flip["s32"]
+
+
+@pytest.mark.parametrize("q", QS)
 def test_unsigned_equals_signed_when_outlier_negative(q):
     W = random_groups(400, 32, 21)
     n_neg = 0
