@@ -22,7 +22,8 @@ got = bench.reduce_max([10.0 * (rank + 1), 5.0 * (rank + 1)], "cpu")
 rate = bench.job_rate(1e6, ws, 4, got[0])
 # the reference arm: rank 0 alone runs and prints; the others exit quietly
 buf = io.StringIO()
-args = type("A", (), dict(steps=1, warmup=0, ref_seconds=0.05))()
+# one core: a spawned oracle pool would re-run this script's top level
+args = type("A", (), dict(steps=1, warmup=0, ref_seconds=0.05, cpu_cores=1))()
 with contextlib.redirect_stdout(buf):
     os.environ["RANK"], os.environ["WORLD_SIZE"] = str(rank), str(ws)
     bench.run_reference(args)
@@ -55,3 +56,20 @@ def test_two_gloo_ranks(tmp_path):
     assert line["cpu_baseline"]["kind"] == "oracle"
     assert line["e2e"]["h2d_bytes_per_step"] == 0
     assert outs[1]["ref"] == ""
+
+
+def test_reference_arm_on_several_host_cores():
+    """The reference arm as the driver launches it: the unchanged oracle in
+    two spawned processes; the line reports the cores it used and the
+    single-process rate beside the total."""
+    out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+                          "--steps", "1", "--warmup", "0", "--ref-seconds", "0.5",
+                          "--cpu-cores", "2"],
+                         cwd=ROOT, capture_output=True, text=True, timeout=300)
+    assert out.returncode == 0, out.stderr[-2000:]
+    line = json.loads(out.stdout.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["value"] > 0
+    cb = line["cpu_baseline"]
+    assert cb["cores"] == 2 and cb["kind"] == "oracle"
+    assert 0 < cb["single_core_value"] <= cb["value"] * 1.01
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
