@@ -354,7 +354,13 @@ def run_ours(args):
                 "mean_launch_us": round(tv / K / wl.gemv_launches * 1e3, 3)}
     cpu = None  # the oracle baseline runs on rank 0 of a single-GPU run only
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(wl, seconds=args.cpu_seconds, cores=args.cpu_cores or host_cores())
+        try:
+            cpu = cpu_baseline(wl, seconds=args.cpu_seconds,
+                               cores=args.cpu_cores or host_cores())
+        except Exception as e:  # noqa: BLE001 - the pool failed mid-run: one process
+            print(f"oracle baseline on several cores failed ({e!r}); timing one process",
+                  file=sys.stderr, flush=True)
+            cpu = cpu_baseline(wl, seconds=args.cpu_seconds, cores=1)
     if rank == 0:
         line = {
             "metric": METRIC, "value": round(gemv_gbs, 1), "unit": "GB/s", "n_gpus": ws,
@@ -464,12 +470,25 @@ def _oracle_gemv_worker(job):
 
 def oracle_pool(cores: int):
     """A pool of `cores` spawned processes for the oracle baseline (spawned,
-    so none inherits CUDA state), or None for one core."""
+    so none inherits CUDA state), or None for one core or when the host
+    cannot start one (the caller then measures one process and reports
+    cores = 1)."""
     if cores <= 1:
         return None
     import multiprocessing as mp
 
-    return mp.get_context("spawn").Pool(cores)
+    try:
+        pool = mp.get_context("spawn").Pool(cores)
+        pool.map(_noop, range(cores))
+        return pool
+    except Exception as e:  # noqa: BLE001 - reported, then one process
+        print(f"oracle baseline: no process pool ({e!r}); timing one process",
+              file=sys.stderr, flush=True)
+        return None
+
+
+def _noop(i):
+    return i
 
 
 def oracle_gemv_rate_cores(pool, cores, codes, scales, n_rows, k, q, xbits, seconds):
@@ -504,6 +523,8 @@ def cpu_baseline(wl, seconds: float, cores: int):
     scales = qt.scales[:4096].cpu().numpy().view(np.uint16)
     xbits = wl.x[k].cpu().view(wl.torch.int16).numpy().view(np.uint16)
     pool = oracle_pool(cores)
+    if pool is None:
+        cores = 1
     try:
         gbs, gbs1, rows, el = oracle_gemv_rate_cores(pool, cores, codes, scales, codes.shape[0],
                                                      k, 4, xbits, seconds)
@@ -537,6 +558,8 @@ def run_reference(args):
     per_step = max(0.5, args.ref_seconds)
     cores = getattr(args, "cpu_cores", 0) or host_cores()
     pool = oracle_pool(cores)
+    if pool is None:
+        cores = 1
     try:
         for _ in range(args.warmup):
             oracle_gemv_rate_cores(pool, cores, *packed[4], rows, k, 4, xbits, 0.05)
