@@ -162,7 +162,6 @@ size_t sss_workspace_bytes(const sss_qtensor_t* qt, int64_t m_or_batch, int32_t 
 sss_status_t sss_gemv(const sss_qtensor_t* qt, const uint16_t* x_bf16, int32_t batch,
                       float* y, void* workspace, size_t ws_bytes,
                       uint32_t* dev_status, void* stream) {
-  (void)dev_status;
   sss_status_t st = check_tensor(qt);
   if (st != SSS_OK) return st;
   if (batch < 1 || batch > 16) return SSS_E_ARG;
@@ -179,6 +178,9 @@ sss_status_t sss_gemv(const sss_qtensor_t* qt, const uint16_t* x_bf16, int32_t b
                   cudaMemsetAsync(y, 0, sizeof(float) * static_cast<size_t>(batch) * qt->n,
                                   static_cast<cudaStream_t>(stream)));
   }
+  // batch 1: the streaming kernel; batch 2..16: the batched kernel (fp16
+  // weight operand); shapes neither takes (k not a multiple of 256,
+  // unaligned buffers): the general kernel
   if (batch == 1 && gemv_stream_eligible(*qt, x_bf16)) {
     const sss_qtensor_t* one[1] = {qt};
     float* yy[1] = {y};
