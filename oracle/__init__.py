@@ -21,6 +21,10 @@ computes, with the passage of the paper it follows:
 * ``matmul_f64`` / ``gemv`` -- the fp64 reference y = x W^T over the
   dequantised weights.
 * ``f32_to_f16`` / ``f16_to_f32`` -- IEEE binary16 from its definition.
+* ``quantize_act_q8`` / ``gemv_q8`` -- the dynamic Q8_0 (narrow-range 8-bit,
+  blocks of 32) activation quantizer the paper pairs with the weight formats
+  (Sec. 5 "Composition with PTQ methods", Appendix C "Algorithm details"),
+  and the fp64 GEMV over dequantised weights and activations.
 
 Every function of the oracle is pinned by ``tests/test_oracle_pins.py``
 against the paper's theorems, closed forms and brute force; nothing in it is
@@ -118,6 +122,10 @@ def lib():
             L.orc_matmul_f64.restype = None
             L.orc_gemv.argtypes = [vp, vp, vp, i64, i64, i32, i32, i32, vp, i64, vp]
             L.orc_gemv.restype = None
+            L.orc_quantize_act_q8.argtypes = [vp, i64, i64, vp, vp]
+            L.orc_quantize_act_q8.restype = i32
+            L.orc_gemv_q8.argtypes = [vp, vp, vp, i64, i64, i32, i32, i32, vp, vp, i64, vp]
+            L.orc_gemv_q8.restype = None
         return _lib
 
 
@@ -246,4 +254,37 @@ def gemv(codes, scales, mins, n: int, k: int, q: int, g: int, grid: int,
     y = np.zeros((nb, n), np.float64)
     lib().orc_gemv(_p(codes), _p(scales), _p(mins), n, k, q, g, grid, _p(x), nb,
                    _p(y))
+    return y
+
+
+def quantize_act_q8(x_bf16):
+    """Q8_0 activations: per block of 32, d = fl32(max|x|/127), q = clip(RNE(x/d),
+    -127, 127), stored fp16 d.  x as bf16 bits [nb, k] (k % 32 == 0).
+    Returns (q int8 [nb, k], d uint16 [nb, k/32] fp16 bits, flags)."""
+    x = np.ascontiguousarray(x_bf16, np.uint16)
+    if x.ndim == 1:
+        x = x[None, :]
+    nb, k = x.shape
+    assert k % 32 == 0
+    q = np.zeros((nb, k), np.int8)
+    d = np.zeros((nb, k // 32), np.uint16)
+    flags = lib().orc_quantize_act_q8(_p(x), nb, k, _p(q), _p(d))
+    return q, d, int(flags)
+
+
+def gemv_q8(codes, scales, mins, n: int, k: int, q: int, g: int, grid: int,
+            xq, xd) -> np.ndarray:
+    """fp64 decode GEMV over the packed weights and Q8_0 activations
+    (xq int8 [nb, k], xd fp16 bits [nb, k/32]); y [nb, n]."""
+    codes = np.ascontiguousarray(codes, np.uint8)
+    scales = np.ascontiguousarray(scales, np.uint16)
+    mins = None if mins is None else np.ascontiguousarray(mins, np.uint16)
+    xq = np.ascontiguousarray(xq, np.int8)
+    xd = np.ascontiguousarray(xd, np.uint16)
+    if xq.ndim == 1:
+        xq, xd = xq[None, :], xd[None, :]
+    nb = xq.shape[0]
+    y = np.zeros((nb, n), np.float64)
+    lib().orc_gemv_q8(_p(codes), _p(scales), _p(mins), n, k, q, g, grid, _p(xq), _p(xd),
+                      nb, _p(y))
     return y

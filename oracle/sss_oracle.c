@@ -346,3 +346,61 @@ void orc_gemv(const uint8_t* codes, const uint16_t* scales,
   free(yr);
   free(row);
 }
+
+/* ------------------------------------------------------------------------ */
+/* Q8_0 activations (narrow range, blocks of 32)                            */
+/* ------------------------------------------------------------------------ */
+
+int32_t orc_quantize_act_q8(const uint16_t* x_bf16, int64_t nb, int64_t k,
+                            int8_t* q, uint16_t* d16) {
+  int32_t flags = 0;
+  const int64_t nblk = k / 32;
+  for (int64_t b = 0; b < nb; ++b) {
+    for (int64_t j = 0; j < nblk; ++j) {
+      const uint16_t* xs = x_bf16 + b * k + j * 32;
+      int8_t* qs = q + b * k + j * 32;
+      float x[32];
+      float M = 0.0f;
+      int bad = 0;
+      for (int i = 0; i < 32; ++i) {
+        x[i] = orc_bf16_to_f32(xs[i]);
+        if (isnan(x[i]) || isinf(x[i])) bad = 1;
+        const float a = fabsf(x[i]);
+        if (a > M) M = a;
+      }
+      if (bad || M == 0.0f) {
+        for (int i = 0; i < 32; ++i) qs[i] = 0;
+        d16[b * nblk + j] = 0;
+        if (bad) flags |= ORC_FLAG_NONFINITE;
+        continue;
+      }
+      const float d = M / 127.0f; /* one IEEE fp32 division */
+      for (int i = 0; i < 32; ++i)
+        qs[i] = (int8_t)clampi((int32_t)orc_rne_quotient(x[i], d), -127, 127);
+      const uint16_t h = orc_f32_to_f16(d);
+      if ((h & 0x7fffu) == 0x7c00u) flags |= ORC_FLAG_RANGE;
+      d16[b * nblk + j] = h;
+    }
+  }
+  return flags;
+}
+
+void orc_gemv_q8(const uint8_t* codes, const uint16_t* scales,
+                 const uint16_t* mins, int64_t n, int64_t k, int32_t q,
+                 int32_t g, int32_t grid, const int8_t* xq,
+                 const uint16_t* xd16, int64_t nb, double* y) {
+  float* row = (float*)malloc((size_t)k * sizeof(float));
+  for (int64_t j = 0; j < n; ++j) {
+    orc_dequantize_rows(codes, scales, mins, n, k, q, g, grid, j, 1, row);
+    for (int64_t b = 0; b < nb; ++b) {
+      double acc = 0.0;
+      for (int64_t i = 0; i < k; ++i) {
+        const double xh = (double)orc_f16_to_f32(xd16[b * (k / 32) + i / 32]) *
+                          (double)xq[b * k + i];
+        acc += (double)row[i] * xh;
+      }
+      y[b * n + j] = acc;
+    }
+  }
+  free(row);
+}

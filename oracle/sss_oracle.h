@@ -113,6 +113,29 @@ void orc_gemv(const uint8_t* codes, const uint16_t* scales,
               const uint16_t* mins, int64_t n, int64_t k, int32_t q, int32_t g,
               int32_t grid, const uint16_t* x_bf16, int64_t nb, double* y);
 
+/* Dynamic Q8_0 activation quantization, the narrow-range 8-bit quantizer
+ * the paper pairs with the few-bit weight formats at inference (Sec. 5,
+ * "Composition with PTQ methods"; Appendix C, "Algorithm details"): the
+ * alphabet {-K..K}, K = 2^(8-1) - 1 = 127, one scale per block of 32
+ * consecutive activations of a token (the GGUF block).  Per block:
+ *   M = max_i |x_i|;  d = fl32(M / 127);
+ *   q_i = clip(RNE(x_i / d), -127, 127) of the exact quotient;
+ *   stored scale d16 = fp16(d).  An all-zero block gives d = 0, q = 0.
+ * x given as bf16 bits [nb][k], k % 32 == 0; q int8 [nb][k]; d16
+ * [nb][k/32].  Returns ORC_FLAG_NONFINITE if an activation is NaN/Inf
+ * (that block's outputs are q = 0, d16 = +0) and ORC_FLAG_RANGE if a
+ * stored d16 is infinite. */
+int32_t orc_quantize_act_q8(const uint16_t* x_bf16, int64_t nb, int64_t k,
+                            int8_t* q, uint16_t* d16);
+
+/* The decode GEMV with Q8_0 activations: y[b][j] = sum_k w^[j][k] * x^[b][k]
+ * in fp64, where w^ is the dequantised weight (orc_dequantize) and
+ * x^ = f16(d) * q the dequantised activation.  y fp64 [nb][n]. */
+void orc_gemv_q8(const uint8_t* codes, const uint16_t* scales,
+                 const uint16_t* mins, int64_t n, int64_t k, int32_t q,
+                 int32_t g, int32_t grid, const int8_t* xq,
+                 const uint16_t* xd16, int64_t nb, double* y);
+
 #ifdef __cplusplus
 }
 #endif

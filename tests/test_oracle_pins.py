@@ -529,3 +529,122 @@ def test_extreme_magnitudes_still_round_to_nearest(q, e):
                 continue
             for j in range(32):
                 assert r["c"][j] == nearest_index(F(float(w[j])), F(0), s, A)
+
+
+# --------------------------------------------------------------------------
+# Q8_0 activations (narrow range, blocks of 32): the runtime pairing of the
+# weight formats (Sec. 5 "Composition with PTQ methods", Appendix C
+# "Algorithm details")
+# --------------------------------------------------------------------------
+
+def _q8_hand_blocks():
+    for line in open(os.path.join(GOLDEN, "q8_act_blocks.txt")):
+        line = line.strip()
+        if not line or line.startswith("#"):
+            continue
+        f = [v.strip() for v in line.split("|")]
+        x = np.zeros(32, np.float32)
+        xs = [float(v) for v in f[0].split()]
+        x[:len(xs)] = xs
+        q = np.zeros(32, np.int8)
+        qs = [int(v) for v in f[1].split()]
+        q[:len(qs)] = qs
+        yield x, q, int(f[2], 16)
+
+
+def test_q8_hand_worked_blocks():
+    blocks = list(_q8_hand_blocks())
+    assert len(blocks) == 4
+    for x, q_want, d_want in blocks:
+        xb = inputs.f32_to_bf16_bits(x)
+        assert np.array_equal(inputs.bf16_bits_to_f32(xb), x)  # exact bf16 values
+        q, d, flags = oracle.quantize_act_q8(xb[None, :])
+        assert flags == 0
+        assert np.array_equal(q[0], q_want)
+        assert int(d[0, 0]) == d_want
+
+
+def _q8_blocks(rng, count):
+    """bf16 blocks of 32: normal, heavy-tailed, tiny, huge and tie-rich."""
+    out = []
+    for i in range(count):
+        kind = i % 5
+        if kind == 0:
+            v = rng.standard_normal(32)
+        elif kind == 1:
+            v = rng.standard_t(3, 32) * 10.0
+        elif kind == 2:
+            v = rng.standard_normal(32) * 1e-30
+        elif kind == 3:
+            v = rng.standard_normal(32) * 1e30
+        else:  # multiples of M/254 hit half-integer quotients
+            v = rng.integers(-254, 255, 32) * 0.5
+        out.append(inputs.f32_to_bf16_bits(v.astype(np.float32)))
+    return np.stack(out)
+
+
+def test_q8_codes_are_nearest_narrow_grid_points():
+    rng = np.random.default_rng(8)
+    xb = _q8_blocks(rng, 400)
+    q, d16, flags = oracle.quantize_act_q8(xb.reshape(1, -1))
+    # the huge blocks' scales overflow fp16 (flagged); their codes still
+    # follow the fp32 scale
+    assert flags == oracle.FLAG_RANGE
+    q = q.reshape(-1, 32)
+    x = inputs.bf16_bits_to_f32(xb)
+    for i in range(x.shape[0]):
+        M = float(np.max(np.abs(x[i])))
+        d = F(float(np.float32(M) / np.float32(127.0)))  # fl32(M / 127)
+        for j in range(32):
+            t = F(float(x[i, j])) / d
+            lo = t.numerator // t.denominator
+            frac = t - lo
+            want = lo + 1 if frac > F(1, 2) or (frac == F(1, 2) and lo % 2 == 1) else lo
+            want = max(-127, min(127, want))
+            assert q[i, j] == want, (i, j)
+        # the block maximum lands on +-127, and -128 never appears
+        jm = int(np.argmax(np.abs(x[i])))
+        assert abs(int(q[i, jm])) == 127
+        assert int(q[i].min()) >= -127
+
+
+def test_q8_is_odd_and_its_error_is_bounded():
+    rng = np.random.default_rng(9)
+    xb = _q8_blocks(rng, 200).reshape(1, -1)
+    q, d16, _ = oracle.quantize_act_q8(xb)
+    qn, dn, _ = oracle.quantize_act_q8(xb ^ np.uint16(0x8000))  # -x
+    assert np.array_equal(qn, -q) and np.array_equal(dn, d16)
+    x = inputs.bf16_bits_to_f32(xb).reshape(-1, 32).astype(np.float64)
+    qf = q.reshape(-1, 32).astype(np.float64)
+    M = np.abs(x).max(axis=1)
+    d32 = (M.astype(np.float32) / np.float32(127.0)).astype(np.float64)
+    dh = np.array([oracle.f16_to_f32(int(v)) for v in d16.ravel()], np.float64)
+    assert np.all(np.abs(x - d32[:, None] * qf) <= d32[:, None] / 2 * (1 + 1e-12))
+    assert np.array_equal(dh, np.array([oracle.f16_to_f32(oracle.f32_to_f16(float(v)))
+                                        for v in d32]))
+
+
+def test_q8_flags():
+    x = np.zeros((1, 64), np.float32)
+    x[0, 3] = np.inf
+    q, d, flags = oracle.quantize_act_q8(inputs.f32_to_bf16_bits(x))
+    assert flags & oracle.FLAG_NONFINITE
+    assert not q[0, :32].any() and d[0, 0] == 0
+    y = np.zeros((1, 32), np.float32)
+    y[0, 0] = 3.0e38  # d = 2.4e36 overflows fp16
+    q, d, flags = oracle.quantize_act_q8(inputs.f32_to_bf16_bits(y))
+    assert flags & oracle.FLAG_RANGE and (int(d[0, 0]) & 0x7fff) == 0x7c00 and q[0, 0] == 127
+
+
+@pytest.mark.parametrize("grid", [oracle.GRID_SIGNED_SYM, oracle.GRID_ASYM])
+def test_gemv_q8_is_matmul_of_dequantised_operands(grid):
+    n, k, q, g = 24, 128, 4, 32
+    W = inputs.student_t_weights(n, k, 77)
+    codes, scales, mins, _, _ = oracle.quantize(W, q, g, grid)
+    xb = inputs.normal_bf16_bits((3, k), 78)
+    xq, xd, _ = oracle.quantize_act_q8(xb)
+    y = oracle.gemv_q8(codes, scales, mins, n, k, q, g, grid, xq, xd)
+    What = oracle.dequantize(codes, scales, mins, n, k, q, g, grid).astype(np.float64)
+    dh = np.array([[oracle.f16_to_f32(int(v)) for v in row] for row in xd], np.float64)
+    xh = xq.astype(np.float64) * np.repeat(dh, 32, axis=1)
+    np.testing.assert_allclose(y, xh @ What.T, rtol=1e-12, atol=1e-12)
