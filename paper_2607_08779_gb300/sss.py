@@ -126,6 +126,46 @@ def _check(fn: str, st: int):
         raise SssError(fn, st, L.sss_last_error().decode())
 
 
+def _need(fn: str, name: str, t, dtype, numel=None, optional=False):
+    """The C ABI takes bare device pointers: check here what a pointer cannot
+    carry (its dtype, a dense layout, its element count) and raise
+    SssError(SSS_E_ARG) before the call; _on_device checks the memory."""
+    if t is None:
+        if optional:
+            return
+        raise SssError(fn, 1, f"{name} is required")
+    if t.dtype != dtype:
+        raise SssError(fn, 1, f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise SssError(fn, 1, f"{name} must be contiguous")
+    if numel is not None and t.numel() != numel:
+        raise SssError(fn, 1, f"{name} holds {t.numel()} elements, expected {numel}")
+
+
+def _on_device(fn: str, **tensors):
+    """Every given tensor (None skipped) lives in CUDA device memory."""
+    for name, t in tensors.items():
+        if t is not None and not getattr(t, "is_cuda", False):
+            raise SssError(fn, 1, f"{name} must be a CUDA tensor")
+
+
+def _need_qtensor(fn: str, qt: "QTensor"):
+    import torch
+
+    ng = qt.k // qt.group if qt.group > 0 else 0
+    _need(fn, "codes", qt.codes, torch.uint8, qt.n * qt.k * qt.q // 8)
+    _need(fn, "scales", qt.scales, torch.int16, qt.n * ng)
+    _need(fn, "mins", qt.mins, torch.int16, qt.n * ng, optional=qt.grid != GRID_ASYM)
+
+
+def _need_status(fn: str, dev_status):
+    import torch
+
+    _need(fn, "dev_status", dev_status, torch.int32, optional=True)
+    if dev_status is not None and dev_status.numel() < 1:
+        raise SssError(fn, 1, "dev_status must hold one int32")
+
+
 @dataclass
 class QTensor:
     """A packed weight tensor: torch device buffers plus its shape metadata."""
@@ -180,9 +220,20 @@ def sss_status_string(status: int) -> str:
 def sss_quantize(w, q: int, group: int, grid: int, out: Optional[QTensor] = None,
                  clip_counts=None, dev_status=None, stream=None) -> QTensor:
     """Quantize fp32 weights w [n, k] (CUDA tensor) into a packed QTensor."""
+    import torch
+
     n, k = w.shape
+    _need("sss_quantize", "w", w, torch.float32)
     if out is None:
         out = empty_qtensor(n, k, q, group, grid, device=w.device)
+    if (out.n, out.k, out.q, out.group, out.grid) != (n, k, q, group, grid):
+        raise SssError("sss_quantize", 1, "out does not match w's shape, q, group and grid")
+    _need_qtensor("sss_quantize", out)
+    if clip_counts is not None and group > 0:
+        _need("sss_quantize", "clip_counts", clip_counts, torch.uint8, n * (k // group) * 2)
+    _need_status("sss_quantize", dev_status)
+    _on_device("sss_quantize", w=w, codes=out.codes, scales=out.scales, mins=out.mins,
+               clip_counts=clip_counts, dev_status=dev_status)
     d = out.desc()
     st = load().sss_quantize(_ptr(w), ctypes.byref(d), _ptr(clip_counts), _ptr(dev_status),
                              _stream(stream))
@@ -196,6 +247,11 @@ def sss_dequantize(qt: QTensor, out=None, out_dtype: int = OUT_F32, stream=None)
     if out is None:
         dt = {OUT_F32: torch.float32, OUT_F16: torch.float16, OUT_BF16: torch.bfloat16}[out_dtype]
         out = torch.empty((qt.n, qt.k), dtype=dt, device=qt.codes.device)
+    _need_qtensor("sss_dequantize", qt)
+    want = {OUT_F32: torch.float32, OUT_F16: torch.float16, OUT_BF16: torch.bfloat16}.get(out_dtype)
+    if want is not None:
+        _need("sss_dequantize", "out", out, want, qt.n * qt.k)
+    _on_device("sss_dequantize", codes=qt.codes, scales=qt.scales, mins=qt.mins, out=out)
     d = qt.desc()
     st = load().sss_dequantize(ctypes.byref(d), _ptr(out), out_dtype, _stream(stream))
     _check("sss_dequantize", st)
@@ -207,8 +263,15 @@ def sss_gemv(qt: QTensor, x, y=None, workspace=None, dev_status=None, stream=Non
     import torch
 
     batch = x.shape[0] if x.dim() == 2 else 1
+    _need("sss_gemv", "x", x, torch.bfloat16, batch * qt.k)
     if y is None:
         y = torch.empty((batch, qt.n), dtype=torch.float32, device=x.device)
+    _need("sss_gemv", "y", y, torch.float32, batch * qt.n)
+    _need_qtensor("sss_gemv", qt)
+    _need("sss_gemv", "workspace", workspace, torch.uint8, optional=True)
+    _need_status("sss_gemv", dev_status)
+    _on_device("sss_gemv", x=x, y=y, codes=qt.codes, scales=qt.scales, mins=qt.mins,
+               workspace=workspace, dev_status=dev_status)
     d = qt.desc()
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     st = load().sss_gemv(ctypes.byref(d), _ptr(x), batch, _ptr(y), _ptr(workspace), ws_bytes,
@@ -223,6 +286,16 @@ def sss_gemv_multi(qts, x, ys=None, flags: int = 0, dev_status=None, stream=None
 
     if ys is None:
         ys = [torch.empty((qt.n,), dtype=torch.float32, device=x.device) for qt in qts]
+    if len(ys) != len(qts):
+        raise SssError("sss_gemv_multi", 1, "one output per matrix")
+    for qt, y in zip(qts, ys):
+        _need("sss_gemv_multi", "x", x, torch.bfloat16, qt.k)
+        _need("sss_gemv_multi", "y", y, torch.float32, qt.n)
+        _need_qtensor("sss_gemv_multi", qt)
+    _need_status("sss_gemv_multi", dev_status)
+    _on_device("sss_gemv_multi", x=x, dev_status=dev_status)
+    for qt, y in zip(qts, ys):
+        _on_device("sss_gemv_multi", y=y, codes=qt.codes, scales=qt.scales, mins=qt.mins)
     descs = [qt.desc() for qt in qts]
     parr = (ctypes.POINTER(QTensorDesc) * len(qts))(*[ctypes.pointer(d) for d in descs])
     yarr = (ctypes.c_void_p * len(qts))(*[_ptr(y) for y in ys])
@@ -237,8 +310,15 @@ def sss_gemm(qt: QTensor, x, y=None, workspace=None, dev_status=None, stream=Non
     import torch
 
     m = x.shape[0]
+    _need("sss_gemm", "x", x, torch.bfloat16, m * qt.k)
     if y is None:
         y = torch.empty((m, qt.n), dtype=torch.float32, device=x.device)
+    _need("sss_gemm", "y", y, torch.float32, m * qt.n)
+    _need_qtensor("sss_gemm", qt)
+    _need("sss_gemm", "workspace", workspace, torch.uint8, optional=True)
+    _need_status("sss_gemm", dev_status)
+    _on_device("sss_gemm", x=x, y=y, codes=qt.codes, scales=qt.scales, mins=qt.mins,
+               workspace=workspace, dev_status=dev_status)
     d = qt.desc()
     if workspace is None:
         need = int(load().sss_workspace_bytes(ctypes.byref(d), m, OP_GEMM))
@@ -254,6 +334,15 @@ def sss_gemm(qt: QTensor, x, y=None, workspace=None, dev_status=None, stream=Non
 def sss_gemm_noalloc(qt: QTensor, x, y, dev_status=None, stream=None):
     """sss_gemm with the library's static scratch instead of a workspace;
     `y` [m, n] fp32 must be given (the call allocates nothing)."""
+    import torch
+
+    m = x.shape[0]
+    _need("sss_gemm_noalloc", "x", x, torch.bfloat16, m * qt.k)
+    _need("sss_gemm_noalloc", "y", y, torch.float32, m * qt.n)
+    _need_qtensor("sss_gemm_noalloc", qt)
+    _need_status("sss_gemm_noalloc", dev_status)
+    _on_device("sss_gemm_noalloc", x=x, y=y, codes=qt.codes, scales=qt.scales, mins=qt.mins,
+               dev_status=dev_status)
     d = qt.desc()
     st = load().sss_gemm_noalloc(ctypes.byref(d), _ptr(x), x.shape[0], _ptr(y),
                                  _ptr(dev_status), _stream(stream))

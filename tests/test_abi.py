@@ -79,3 +79,42 @@ def test_gemv_gemm_argument_checks():
     assert L.sss_gemv(ctypes.byref(d0), x, 1, y, None, 0, None, None) == 0
     assert L.sss_gemm(ctypes.byref(d), x, 0, y, None, 0, None, None) == 0
     assert L.sss_quantize(ctypes.c_void_p(4096), ctypes.byref(_desc(n=0)), None, None, None) == 0
+
+
+def test_binding_checks_what_a_pointer_cannot_carry():
+    """The Python binding rejects tensors the C ABI would misread (wrong
+    dtype, strided, wrong element count, host memory) with SSS_E_ARG before
+    any call into the library."""
+    torch = pytest.importorskip("torch")
+    n, k = 16, 256
+    qt = sss.empty_qtensor(n, k, 4, 32, sss.GRID_SIGNED_SYM, device="cpu")
+    x = torch.zeros((2, k), dtype=torch.bfloat16)
+    y = torch.zeros((2, n), dtype=torch.float32)
+    cases = [
+        (lambda: sss.sss_gemv(qt, x.float(), y=y), "bfloat16"),
+        (lambda: sss.sss_gemv(qt, torch.zeros((k, 2), dtype=torch.bfloat16).t(), y=y),
+         "contiguous"),
+        (lambda: sss.sss_gemv(qt, torch.zeros((2, 128), dtype=torch.bfloat16), y=y),
+         "elements"),
+        (lambda: sss.sss_gemv(qt, x, y=torch.zeros((2, n + 1))), "elements"),
+        (lambda: sss.sss_gemv(qt, x, y=y), "CUDA"),
+        (lambda: sss.sss_gemv_multi([qt], x[0], ys=[y[0].double()]), "float32"),
+        (lambda: sss.sss_gemm(qt, x, y=y.int()), "float32"),
+        (lambda: sss.sss_quantize(torch.zeros((n, k), dtype=torch.float64), 4, 32,
+                                  sss.GRID_SIGNED_SYM), "float32"),
+        (lambda: sss.sss_quantize(torch.zeros((n, k)), 4, 32, sss.GRID_SIGNED_SYM,
+                                  out=sss.empty_qtensor(n, k, 3, 32, sss.GRID_SIGNED_SYM,
+                                                        device="cpu")), "out"),
+        (lambda: sss.sss_dequantize(qt, out=torch.zeros((n, k), dtype=torch.float16)),
+         "float32"),
+        (lambda: sss.sss_gemm_noalloc(qt, x, y[:1]), "elements"),
+    ]
+    for call, what in cases:
+        with pytest.raises(sss.SssError) as e:
+            call()
+        assert e.value.status == 1 and what in str(e.value), str(e.value)
+    # a min-max tensor needs its mins
+    asym = sss.empty_qtensor(n, k, 4, 32, sss.GRID_ASYM, device="cpu")
+    asym.mins = None
+    with pytest.raises(sss.SssError, match="mins"):
+        sss.sss_gemv(asym, x, y=y)
