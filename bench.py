@@ -910,7 +910,8 @@ def main():
     ap.add_argument("--rows", type=int, default=0, help="micro: override every matrix's rows")
     ap.add_argument("--sweep", choices=["qwen3_quantize", "grids", "margins"],
                     help="measurement sweeps: whole-model quantization of Qwen3-32B shapes, "
-                         "or the unsigned / signed / min-max grid comparison")
+                         "the unsigned / signed / min-max grid comparison, or the "
+                         "cardinality margin against the realised l2 gain")
     args = ap.parse_args()
     if args.sweep == "qwen3_quantize":
         sweep_qwen3_quantize(args)
