@@ -4,13 +4,16 @@
  *
  * Readings of points the paper leaves open (also listed in the design notes):
  *  - Sign tie: when max w == -min w the dominant outlier is ambiguous
- *    ("deterministic tie-breaking", Sec. 3 after eq:sign_rule); we take
+ *    (Sec. 3 after eq:sign_rule asks for a deterministic tie-break but names
+ *    no rule); we take
  *    gamma = +1, the standard convention.
  *  - RTN tie (w/s exactly a half-integer, assumed away in Sec. 4): round
  *    half to even of the EXACT quotient.  The fp64 quotient of two fp32
  *    numbers decides RNE of the exact quotient correctly (see
  *    orc_rne_quotient).
  *  - M == 0: all codes 0 and stored scale +0 (the paper requires M > 0).
+ *    The same holds when alpha = M / 2^(q-1) underflows to zero in fp32
+ *    (M <= 2^(q-151)), where the paper's s != 0 cannot be met.
  *  - Asymmetric grid (eq:minmax): s = fl32(fl32(max-min)/(2^q-1)), the code
  *    is RNE(fl32(w-min)/s) clipped to {0..2^q-1}, i.e. eq:quantizer with
  *    z = -min/s written as (w-min)/s; the minimum is stored as fp16 and the
@@ -121,10 +124,15 @@ int32_t orc_quantize_group_gamma(const float* w, int32_t g, int32_t q,
   r.gamma = gamma;
   const int32_t half = 1 << (q - 1);           /* 2^(q-1)              */
   const int32_t amin = -half, amax = half - 1; /* A_q = {-2^(q-1)..2^(q-1)-1} */
-  if (r.M == 0.0f || (r.flags & ORC_FLAG_NONFINITE)) {
+  /* alpha := M / 2^(q-1): exact power-of-two scaling of M, except that a
+   * subnormal M can round it (to zero when M <= 2^(q-151)) */
+  const float alpha = ldexpf(r.M, -(q - 1));
+  if (r.M == 0.0f || alpha == 0.0f || (r.flags & ORC_FLAG_NONFINITE)) {
     /* all-zero group: codes 0, stored scale +0 (reading; the paper assumes
-     * M > 0).  A group holding NaN/Inf is flagged and given the same
-     * placeholder outputs; its content is not meaningful. */
+     * M > 0 and s != 0).  A group whose alpha underflows to zero has no
+     * usable scale and is given the same outputs (reading).  A group
+     * holding NaN/Inf is flagged and given the same placeholder outputs;
+     * its content is not meaningful. */
     r.alpha = 0.0f;
     r.s32 = 0.0f;
     for (int32_t j = 0; j < g; ++j) {
@@ -133,8 +141,7 @@ int32_t orc_quantize_group_gamma(const float* w, int32_t g, int32_t q,
       if (u) u[j] = (uint8_t)half;
     }
   } else {
-    /* alpha := M / 2^(q-1): exact power-of-two scaling of M */
-    r.alpha = ldexpf(r.M, -(q - 1));
+    r.alpha = alpha;
     r.s32 = (float)gamma * r.alpha; /* s := gamma * alpha */
     for (int32_t j = 0; j < g; ++j) {
       /* round-to-nearest of w/s, then clip to A_q (eq:quantizer, z = 0) */

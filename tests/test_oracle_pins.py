@@ -531,6 +531,48 @@ def test_extreme_magnitudes_still_round_to_nearest(q, e):
                 assert r["c"][j] == nearest_index(F(float(w[j])), F(0), s, A)
 
 
+@pytest.mark.parametrize("q", QS)
+def test_underflowed_alpha_is_a_zero_group(q):
+    """alpha = M / 2^(q-1) of a subnormal M is rounded to a multiple of
+    2^-149 (ties to the even multiple), so it is zero exactly when
+    M = j * 2^-149 with j <= 2^(q-2).  Then no scale s != 0 exists
+    (eq:absmax needs s != 0) and the group gets the all-zero group's
+    outputs: every code 0 (stored 2^(q-1)) and a +0 scale, for both signs."""
+    half = 1 << (q - 1)
+    for j in range(1, 4 * half + 1):
+        M = j * 2.0 ** -149
+        for sign in (1.0, -1.0):
+            w = np.zeros(32, np.float32)
+            w[3] = np.float32(sign * M)
+            w[7] = np.float32(-sign * 2.0 ** -149) if j > 1 else 0.0
+            for grid in (oracle.GRID_UNSIGNED_SYM, oracle.GRID_SIGNED_SYM):
+                r = oracle.quantize_group(w, q, grid)
+                if F(j, half) <= F(1, 2):  # alpha rounds to zero
+                    assert r["s32"] == 0.0 and r["s16"] == 0x0000, (j, sign)
+                    assert np.all(r["u"] == half) and np.all(r["c"] == 0)
+                    assert r["flags"] == 0
+                else:
+                    assert r["s32"] != 0.0
+                    s = F(r["s32"])
+                    for e in range(32):
+                        assert r["c"][e] == nearest_index(F(float(w[e])), F(0), s, alphabet(q))
+
+
+@pytest.mark.parametrize("q", QS)
+def test_asym_zero_minimum_is_stored_as_plus_zero(q):
+    """Reading of eq:minmax's stored minimum: a zero minimum is stored as +0
+    (fp16 bits 0x0000), whichever zero the group holds or meets first."""
+    base = np.linspace(0.0, 1.0, 32).astype(np.float32)
+    for zeros in ([-0.0], [-0.0, 0.0], [0.0, -0.0]):
+        w = base.copy()
+        for i, z in enumerate(zeros):
+            w[i] = np.float32(z)
+        assert np.signbit(w[0]) == np.signbit(np.float32(zeros[0]))
+        r = oracle.quantize_group(w, q, oracle.GRID_ASYM)
+        assert r["m16"] == 0x0000, zeros
+        assert r["u"][0] == 0 and r["u"][31] == (1 << q) - 1
+
+
 # --------------------------------------------------------------------------
 # Q8_0 activations (narrow range, blocks of 32): the runtime pairing of the
 # weight formats (Sec. 5 "Composition with PTQ methods", Appendix C
