@@ -36,7 +36,8 @@
  * The stored code is u = c + 2^(q-1) for the symmetric grids (c in the signed
  * alphabet {-2^(q-1) .. 2^(q-1)-1}) and u = c in {0 .. 2^q-1} for ASYM.
  * scales: IEEE fp16 [n][k/group], the signed scale s = gamma*alpha for the
- * symmetric grids (Appendix B.1: "may be negative"), the step for ASYM.
+ * symmetric grids (Appendix B.1 lets the stored scale be negative), the step
+ * for ASYM.
  * mins: fp16 [n][k/group], ASYM only (the stored minimum m; w^ = s*u + m).
  */
 #ifndef SSS_H
@@ -78,8 +79,8 @@ typedef enum { SSS_OUT_F32 = 0, SSS_OUT_F16 = 1, SSS_OUT_BF16 = 2 } sss_dtype_t;
 
 /* A packed weight tensor.  Plain descriptor; the library never frees it. */
 typedef struct {
-  int64_t n;         /* rows (output features), >= 0                                */
-  int64_t k;         /* columns (input features), multiple of `group`             */
+  int64_t n;         /* rows (output features), 0 .. 2^31                           */
+  int64_t k;         /* columns (input features), 0 .. 2^31, multiple of `group`  */
   int32_t q;         /* bits per code: 2, 3 or 4                                   */
   int32_t group;     /* group size along k: 32, 64 or 128                          */
   int32_t grid;      /* sss_grid_t                                                 */
@@ -173,7 +174,9 @@ sss_status_t sss_gemv(const sss_qtensor_t* qt, const uint16_t* x_bf16,
  * sss_gemv_multi -- batch-1 decode GEMV of several packed matrices that
  * share one activation vector (e.g. the q/k/v or gate/up projections of a
  * layer) in one launch: y_j[r] = sum_k w^_j[r][k] * x[k] (same arithmetic as
- * sss_gemv).  The weights are streamed through shared memory by bulk copies.
+ * sss_gemv).  Every lane loads the packed bytes it multiplies straight into
+ * registers (a ring one unit ahead of its use); only the activations are
+ * staged in shared memory.
  *   qts     [in]  count pointers to packed tensors with equal k, q, group and
  *                 grid; codes, scales (and mins) 16-byte aligned.
  *   ys      [out] count device fp32 pointers, y_j of length qts[j]->n.
@@ -190,15 +193,15 @@ sss_status_t sss_gemv_multi(const sss_qtensor_t* const* qts, float* const* ys,
                             uint32_t* dev_status, void* stream);
 
 /*
- * sss_gemm -- prefill GEMM Y[m][r] = sum_k w^[r][k] * X[m][k] (Appendix B.3,
- * "compute-bound phase dominated by matrix multiplications"), dequantising
+ * sss_gemm -- prefill GEMM Y[m][r] = sum_k w^[r][k] * X[m][k] (Appendix B.3;
+ * prefill is the phase where the matrix products set the time), dequantising
  * weight tiles on chip and accumulating on the tcgen05 tensor cores in fp32
  * (tensor memory).  Tile operands are fp16: w^ rounded to fp16 and X
  * converted from bf16 (exact for 2^-17 <= |x| <= 65504).
  *   qt        [in]  packed tensor, symmetric grids or ASYM; k % 64 == 0;
  *                   codes 16-byte aligned.
  *   x_bf16    [in]  device bf16 [m][k], 16-byte aligned.
- *   m         [in]  >= 0 tokens.
+ *   m         [in]  0 .. 2^24 tokens.
  *   y         [out] device fp32 [m][n], 16-byte aligned, n % 4 == 0.
  *   workspace [in]  as for sss_gemv with SSS_OP_GEMM.
  *   dev_status [out] nullable; SSS_FLAG_TIMEOUT if a bounded wait expired.

@@ -1,8 +1,8 @@
 // gemm.cu -- prefill GEMM over packed q-bit codes on the 5th-generation
 // tensor cores (sm_103a: tcgen05 + tensor memory + TMA).
 //
-// Y[m][r] = sum_k w^[r][k] X[m][k]; the prefill phase is "a compute-bound
-// phase dominated by matrix multiplications" (Appendix B.2), and the
+// Y[m][r] = sum_k w^[r][k] X[m][k]; in the prefill phase the matrix products
+// set the time (Appendix B.2), and the
 // symmetric formats compute only the integer-code GEMM term of the expansion
 // in Appendix B.3 (the min-max grid adds the per-block minimum).
 //
@@ -486,8 +486,13 @@ __global__ void __launch_bounds__(256)
 // host side
 // ---------------------------------------------------------------------------
 
+// bytes of the fp16 copy of X, rounded up to 256; SIZE_MAX when m * k * 2
+// does not fit in size_t (such a call is rejected before it gets here)
 size_t x16_bytes(int64_t m, int64_t k) {
-  return (static_cast<size_t>(m) * static_cast<size_t>(k) * 2 + 255) / 256 * 256;
+  if (m < 0 || k < 0) return SIZE_MAX;
+  const size_t mm = static_cast<size_t>(m), kk = static_cast<size_t>(k);
+  if (kk != 0 && mm > (SIZE_MAX - 255) / 2 / kk) return SIZE_MAX;
+  return (mm * kk * 2 + 255) / 256 * 256;
 }
 
 template <int Q, bool ASYM, int BN>

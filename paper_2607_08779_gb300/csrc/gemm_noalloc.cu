@@ -9,6 +9,7 @@
 // module, so with lazy module loading it takes device memory only once this
 // entry point is first used.
 #include <mutex>
+#include <stdio.h>
 
 #include "sss_internal.cuh"
 
@@ -53,6 +54,9 @@ size_t sss_gemm_noalloc_max_scratch_bytes(void) { return kScratchBytes; }
 sss_status_t sss_gemm_noalloc(const sss_qtensor_t* qt, const uint16_t* x_bf16, int64_t m,
                               float* y, uint32_t* dev_status, void* stream) {
   if (qt == nullptr) return SSS_E_ARG;
+  // sss_gemm itself rejects m outside 0..2^24 with SSS_E_ARG; a larger m
+  // must not reach the size check below as a wrapped byte count
+  if (m < 0 || m > (int64_t{1} << 24)) return SSS_E_ARG;
   const size_t need = sss_workspace_bytes(qt, m, SSS_OP_GEMM);
   if (need > kScratchBytes) {
     sss::set_error_message("sss_gemm_noalloc: the fp16 copy of X needs more than the "
@@ -62,7 +66,11 @@ sss_status_t sss_gemm_noalloc(const sss_qtensor_t* qt, const uint16_t* x_bf16, i
   cudaError_t err = cudaSuccess;
   void* ws = scratch_ptr(&err);
   if (ws == nullptr) {
-    sss::set_error_message("sss_gemm_noalloc: cudaGetSymbolAddress of the static scratch failed");
+    char msg[200];
+    snprintf(msg, sizeof msg,
+             "sss_gemm_noalloc: cudaGetSymbolAddress of the static scratch failed: %s (%d)",
+             cudaGetErrorString(err), static_cast<int>(err));
+    sss::set_error_message(msg);
     return SSS_E_CUDA;
   }
   return sss_gemm(qt, x_bf16, m, y, ws, kScratchBytes, dev_status, stream);

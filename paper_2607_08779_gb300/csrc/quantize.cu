@@ -164,9 +164,11 @@ __global__ void __launch_bounds__(kQuantThreads)
       // M = ||w||_inf; gamma* = -sign(w_i*): the outlier is positive iff
       // max w > -min w (a tie keeps gamma = +1).
       const float M = fmaxf(mx, -mn);
-      const bool zero = (M == 0.f) || bad;
       const float gamma = (GRID == SSS_GRID_SIGNED_SYM && mx > -mn) ? -1.f : 1.f;
       const float alpha = __fmul_rn(M, 1.0f / HALF);  // M * 2^-(q-1), exact unless subnormal
+      // an alpha that underflows to zero (M <= 2^(q-151)) leaves no scale
+      // s != 0: such a group is quantized like an all-zero group
+      const bool zero = (alpha == 0.f) || bad;
       const float s = zero ? 0.f : gamma * alpha;
       if (zero) {
 #pragma unroll

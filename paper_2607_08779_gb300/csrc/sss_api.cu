@@ -19,6 +19,12 @@ void set_error(const char* what, cudaError_t e) {
            cudaGetErrorString(e), static_cast<int>(e));
 }
 
+// largest n or k a tensor may have, and the most tokens of one sss_gemm:
+// keeps every size product of the launchers far inside int64/size_t and the
+// GEMM's token-tile grid dimension inside its 65535 limit
+constexpr int64_t kMaxDim = int64_t{1} << 31;
+constexpr int64_t kMaxTokens = int64_t{1} << 24;
+
 bool aligned(const void* p, size_t a) {
   return (reinterpret_cast<uintptr_t>(p) % a) == 0;
 }
@@ -30,6 +36,7 @@ sss_status_t check_tensor(const sss_qtensor_t* t) {
   if (t->grid < SSS_GRID_UNSIGNED_SYM || t->grid > SSS_GRID_ASYM) return SSS_E_ARG;
   if (t->reserved != 0) return SSS_E_ARG;
   if (t->n < 0 || t->k < 0) return SSS_E_ARG;
+  if (t->n > kMaxDim || t->k > kMaxDim) return SSS_E_ARG;
   if (t->k % t->group != 0) return SSS_E_ARG;
   if (t->n > 0 && t->k > 0) {
     if (t->codes == nullptr || t->scales == nullptr) return SSS_E_ARG;
@@ -230,7 +237,7 @@ sss_status_t sss_gemm(const sss_qtensor_t* qt, const uint16_t* x_bf16, int64_t m
                       uint32_t* dev_status, void* stream) {
   sss_status_t st = check_tensor(qt);
   if (st != SSS_OK) return st;
-  if (m < 0) return SSS_E_ARG;
+  if (m < 0 || m > kMaxTokens) return SSS_E_ARG;
   if (m == 0 || qt->n == 0) return SSS_OK;
   if (x_bf16 == nullptr || y == nullptr) return SSS_E_ARG;
   if (qt->k % 64 != 0) return SSS_E_UNSUPPORTED;

@@ -87,6 +87,10 @@ def special_groups(g):
     lat2 = rng.integers(-16, 17, g) / 16.0; lat2[1] = -1.0; out.append(lat2)
     for e in (-140, -130, -126, -100, -97, 97, 100, 120):
         out.append(base[1] * 2.0 ** e)              # subnormal / tiny / huge
+    for j in (1, 2, 3, 4, 5):                        # M = j * 2^-149: alpha may round to 0
+        t = np.zeros(g); t[2] = j * 2.0 ** -149; t[9] = -2.0 ** -149
+        out.append(t)
+        out.append(-t)
     out.append(np.full(g, 0.375))                    # constant group
     out.append(base[2] * 1e6)                        # fp16 scale overflow
     return np.stack(out).astype(np.float32)
