@@ -240,6 +240,24 @@ sss_status_t sss_gemm_noalloc(const sss_qtensor_t* qt, const uint16_t* x_bf16,
                               void* stream);
 size_t sss_gemm_noalloc_max_scratch_bytes(void);
 
+/*
+ * sss_test_set_stall -- test hook for the bounded waits; the paper has no
+ * counterpart.  While a bit below is set, every later launch of that kernel
+ * family leaves one mbarrier one arrive short: the batch-1 GEMV and the
+ * batched GEMV on the first output tile's partial sums (only where a tile's
+ * k-range is split across several warps), the GEMM on the first stage's
+ * weight tile.  The wait on that barrier then runs out after its bound
+ * (about one second), the kernel raises SSS_FLAG_TIMEOUT in dev_status,
+ * lets its own copies and MMAs in flight finish, releases its tensor memory
+ * and returns; its output is incomplete.  Nothing faults or hangs.
+ * mask = 0 (the default) restores normal launches.  Process-wide; affects
+ * launches issued (or captured) after the call on every thread.
+ */
+#define SSS_TEST_STALL_GEMV 0x1u       /* gemv_stream_kernel (sss_gemv batch 1, sss_gemv_multi) */
+#define SSS_TEST_STALL_GEMV_BATCH 0x2u /* gemv_batch_kernel (sss_gemv batch 2..16)             */
+#define SSS_TEST_STALL_GEMM 0x4u       /* gemm_kernel (sss_gemm, sss_gemm_noalloc)             */
+void sss_test_set_stall(uint32_t mask);
+
 #ifdef __cplusplus
 }
 #endif

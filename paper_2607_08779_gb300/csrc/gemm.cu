@@ -247,6 +247,7 @@ struct GemmArgs {
   uint32_t* status;
   int64_t m, n, k;
   int G;
+  int stall;  // test hook: the first stage's weight tile is never announced
 };
 
 template <int BN, int STAGES>
@@ -419,7 +420,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         fence_proxy_async_smem();  // generic-proxy stores -> visible to the tensor core
         __syncwarp();
-        if (lane == 0) mbar_arrive(&full_a[s]);
+        // (sss_test_set_stall: warp 2 leaves the first stage one arrive
+        // short, so the MMA issuer's wait for it runs out)
+        if (lane == 0 && !(a.stall && kb == 0 && warp == 2)) mbar_arrive(&full_a[s]);
         fetch(ring[q0], kb + kDqSets * kPrefetch);
       }
     }
@@ -525,6 +528,7 @@ cudaError_t run_gemm(const sss_qtensor_t& t, const __half* x16, int64_t m, float
   a.n = t.n;
   a.k = t.k;
   a.G = t.group;
+  a.stall = (test_stall_mask() & SSS_TEST_STALL_GEMM) ? 1 : 0;
   dim3 grid(static_cast<unsigned>((t.n + kBM - 1) / kBM), static_cast<unsigned>((m + BN - 1) / BN));
   kern<<<grid, kThreads, S::TOTAL, stream>>>(map, a);
   return cudaGetLastError();

@@ -54,6 +54,7 @@ struct BatchArgs {
   int64_t ntiles;
   int lgkw;        // log2(warps per tile)
   int slab_units;  // units of 256 codes per x slab
+  int stall;       // test hook: the first tile's barrier stays one arrive short
   uint32_t* status;
 };
 
@@ -389,7 +390,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_batch_kernel(const __grid_co
         acc[nb][e] = 0.f;
       }
     __syncwarp();
-    if (lane == 0) bar_arrive(rdy);
+    // (sss_test_set_stall: the last warp leaves the first tile's barrier one
+    // arrive short, so its reducer's wait runs out)
+    if (lane == 0 && !(a.stall && s == 0 && i == 0 && kw == KW - 1)) bar_arrive(rdy);
     if (kw == static_cast<int>(i & (KW - 1))) {
       if (!bar_wait(rdy, use, abort)) ok = false;
       for (int v = lane; v < R * NBC; v += 32) {
@@ -515,6 +518,7 @@ cudaError_t launch_gemv_batch(const sss_qtensor_t& t, const uint16_t* x, int bat
   a.k = t.k;
   a.batch = batch;
   a.status = status;
+  a.stall = (test_stall_mask() & SSS_TEST_STALL_GEMV_BATCH) ? 1 : 0;
   const bool asym = t.grid == SSS_GRID_ASYM;
   switch (t.q) {
     case 2: return asym ? launch_bg<2, true>(t, a, stream) : launch_bg<2, false>(t, a, stream);

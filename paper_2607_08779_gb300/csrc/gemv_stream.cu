@@ -62,6 +62,7 @@ struct StreamArgs {
   int64_t ntiles;
   int lgkw;            // log2(warps per tile)
   int early_weights;   // prefetch weights before the grid-dependency wait
+  int stall;           // test hook: one partial of the first tile is never announced
   uint32_t* status;
 };
 
@@ -330,7 +331,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
       if (!bar_wait(fre, use ^ 1u, abort)) ok = false;
       pb[kw * R + gq] = v[0];
       pb[kw * R + gq + 8] = v[1];
-      bar_arrive(rdy);
+      // (sss_test_set_stall: the last warp's first quad leaves the first
+      // tile's barrier one arrive short, so its reducer's wait runs out)
+      if (!(a.stall && i == 0 && kw == KW - 1 && gq == 0)) bar_arrive(rdy);
     }
     if (kw == static_cast<int>(i & (KW - 1))) {
       if (!bar_wait(rdy, use, abort)) ok = false;
@@ -481,6 +484,7 @@ cudaError_t launch_gemv_stream(const sss_qtensor_t* const* ts, float* const* ys,
   a.x = x;
   a.k = ts[0]->k;
   a.early_weights = (flags & SSS_GEMV_WEIGHTS_READY) ? 1 : 0;
+  a.stall = (test_stall_mask() & SSS_TEST_STALL_GEMV) ? 1 : 0;
   a.status = status;
   for (int j = 0; j < count; ++j) {
     a.job[j].codes = ts[j]->codes;

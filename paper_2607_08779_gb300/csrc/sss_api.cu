@@ -1,6 +1,7 @@
 // sss_api.cu -- the C ABI declared in include/sss.h: synchronous argument
 // validation, dispatch to the kernels' launchers, and error mapping.  No
 // entry point allocates device memory.
+#include <atomic>
 #include <map>
 #include <mutex>
 #include <utility>
@@ -100,6 +101,12 @@ int device_sm_count() {
   return cache[dev];
 }
 
+namespace {
+std::atomic<uint32_t> g_test_stall{0};
+}  // namespace
+
+uint32_t test_stall_mask() { return g_test_stall.load(std::memory_order_relaxed); }
+
 void set_error_message(const char* msg) {
   snprintf(g_last_error, sizeof g_last_error, "%s", msg);
 }
@@ -128,6 +135,11 @@ const char* sss_status_string(sss_status_t s) {
 }
 
 const char* sss_last_error(void) { return g_last_error; }
+
+void sss_test_set_stall(uint32_t mask) {
+  g_test_stall.store(mask & (SSS_TEST_STALL_GEMV | SSS_TEST_STALL_GEMV_BATCH | SSS_TEST_STALL_GEMM),
+                     std::memory_order_relaxed);
+}
 
 sss_status_t sss_quantize(const float* w, const sss_qtensor_t* out,
                           uint8_t* clip_counts, uint32_t* dev_status,

@@ -48,6 +48,10 @@ cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m,
                         float* y, void* workspace, uint32_t* status,
                         cudaStream_t stream);
 
+// The kernel families whose next launches skip one barrier arrive
+// (sss_test_set_stall; 0 in normal use).
+uint32_t test_stall_mask();
+
 // Record a message for sss_last_error() on this thread.
 void set_error_message(const char* msg);
 

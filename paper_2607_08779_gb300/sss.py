@@ -32,10 +32,14 @@ STATUS_NAMES = {0: "SSS_OK", 1: "SSS_E_ARG", 2: "SSS_E_UNSUPPORTED", 3: "SSS_E_A
 
 EXPORTS = ("sss_codes_bytes", "sss_status_string", "sss_last_error", "sss_quantize",
            "sss_dequantize", "sss_gemv", "sss_gemv_multi", "sss_gemm", "sss_workspace_bytes",
-           "sss_gemm_noalloc", "sss_gemm_noalloc_max_scratch_bytes")
+           "sss_gemm_noalloc", "sss_gemm_noalloc_max_scratch_bytes", "sss_test_set_stall")
 
 GEMV_PDL = 0x1
 GEMV_WEIGHTS_READY = 0x2
+
+TEST_STALL_GEMV = 0x1
+TEST_STALL_GEMV_BATCH = 0x2
+TEST_STALL_GEMM = 0x4
 
 
 class SssError(RuntimeError):
@@ -104,6 +108,8 @@ def load(build_if_needed: bool = True):
         L.sss_gemm_noalloc.restype = i32
         L.sss_gemm_noalloc_max_scratch_bytes.argtypes = []
         L.sss_gemm_noalloc_max_scratch_bytes.restype = sz
+        L.sss_test_set_stall.argtypes = [ctypes.c_uint32]
+        L.sss_test_set_stall.restype = None
         _lib = L
         return L
 
@@ -352,3 +358,10 @@ def sss_gemm_noalloc(qt: QTensor, x, y, dev_status=None, stream=None):
 
 def sss_gemm_noalloc_max_scratch_bytes() -> int:
     return int(load().sss_gemm_noalloc_max_scratch_bytes())
+
+
+def sss_test_set_stall(mask: int) -> None:
+    """Test hook of the bounded waits (TEST_STALL_* bits; 0 restores normal
+    launches): later launches of the named kernels leave one barrier one
+    arrive short, so a wait runs out and the kernel raises FLAG_TIMEOUT."""
+    load().sss_test_set_stall(int(mask))

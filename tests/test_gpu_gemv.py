@@ -21,9 +21,11 @@ def run_case(n, k, q, g, grid, batch, seed, rows=None, outliers=True, tol=REL_TO
     qt = qtensor_from_oracle(codes, scales, mins, n, k, q, g, grid)
     xb = x_bits(batch, k, seed + 1)
     x = to_dev(xb.view(np.int16)).view(torch.bfloat16)
-    y = sss.sss_gemv(qt, x)
-    y2 = sss.sss_gemv(qt, x)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    y = sss.sss_gemv(qt, x, dev_status=st)
+    y2 = sss.sss_gemv(qt, x, dev_status=st)
     torch.cuda.synchronize()
+    assert int(st.item()) == 0, f"device status {int(st.item()):#x}"
     assert torch.equal(y, y2), "GEMV is not deterministic"
     y = y.cpu().numpy()
     if rows is None:

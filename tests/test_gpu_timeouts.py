@@ -1,0 +1,123 @@
+"""The bounded waits of the GEMV and GEMM kernels, made to run out.
+
+sss_test_set_stall leaves one mbarrier of the chosen kernel one arrive
+short, so the wait on it expires after its bound (about one second).  The
+call must still return SSS_OK, the device status word must carry
+SSS_FLAG_TIMEOUT, and a normal call right after it must match the oracle:
+the kernel released its tensor memory and the context is still usable.
+Nothing here faults, traps or hangs the GPU.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_util import REL_TOL, qtensor_from_oracle, rel_err_per_row, to_dev, x_bits
+from paper_2607_08779_gb300 import inputs, sss
+
+pytestmark = pytest.mark.gpu
+
+GRID = oracle.GRID_SIGNED_SYM
+
+
+def _packed(n, k, q, g, seed):
+    W = inputs.student_t_weights(n, k, seed)
+    codes, scales, mins, _, _ = oracle.quantize(W, q, g, GRID)
+    return qtensor_from_oracle(codes, scales, mins, n, k, q, g, GRID), (codes, scales, mins)
+
+
+def _x(bits):
+    return to_dev(bits.view(np.int16)).view(torch.bfloat16)
+
+
+def _stalled(mask, call):
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    sss.sss_test_set_stall(mask)
+    try:
+        call(st)  # raises SssError on a non-OK return code
+        torch.cuda.synchronize()
+    finally:
+        sss.sss_test_set_stall(0)
+    return int(st.item())
+
+
+@pytest.mark.parametrize("batch", [1, 4])
+def test_gemv_wait_runs_out_then_recovers(batch):
+    # one 16-row tile whose 4096-code rows are split across all 16 warps of
+    # the CTA, so the partial sums meet behind a barrier
+    n, k, q, g = 16, 4096, 4, 32
+    qt, (codes, scales, mins) = _packed(n, k, q, g, 21)
+    xb = x_bits(batch, k, 5)
+    x = _x(xb)
+    y = torch.empty((batch, n), dtype=torch.float32, device="cuda")
+    mask = sss.TEST_STALL_GEMV if batch == 1 else sss.TEST_STALL_GEMV_BATCH
+    status = _stalled(mask, lambda st: sss.sss_gemv(qt, x, y=y, dev_status=st))
+    assert status & sss.FLAG_TIMEOUT, status
+
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    y = sss.sss_gemv(qt, x, dev_status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    yref = oracle.gemv(codes, scales, mins, n, k, q, g, GRID, xb)
+    assert rel_err_per_row(y.cpu().numpy(), yref).max() <= REL_TOL
+
+
+def test_gemv_multi_wait_runs_out_then_recovers():
+    n, k, q, g = 16, 4096, 3, 32
+    qa, (ca, sa, ma) = _packed(n, k, q, g, 22)
+    qb, (cb, sb, mb) = _packed(n, k, q, g, 23)
+    xb = x_bits(1, k, 6)
+    x = _x(xb)[0]
+    status = _stalled(sss.TEST_STALL_GEMV,
+                      lambda st: sss.sss_gemv_multi([qa, qb], x, dev_status=st,
+                                                    flags=sss.GEMV_PDL | sss.GEMV_WEIGHTS_READY))
+    assert status & sss.FLAG_TIMEOUT, status
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ya, yb = sss.sss_gemv_multi([qa, qb], x, dev_status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    for y, (c, s, m) in ((ya, (ca, sa, ma)), (yb, (cb, sb, mb))):
+        yref = oracle.gemv(c, s, m, n, k, q, g, GRID, xb)
+        assert rel_err_per_row(y.cpu().numpy()[None], yref).max() <= REL_TOL
+
+
+@pytest.mark.parametrize("noalloc", [False, True])
+def test_gemm_wait_runs_out_then_recovers(noalloc):
+    # 16 k-blocks of 64, more than the pipeline's stages, and two token tiles
+    n, k, q, g, m = 256, 1024, 4, 32, 200
+    qt, (codes, scales, mins) = _packed(n, k, q, g, 24)
+    Xb = x_bits(m, k, 7)
+    X = _x(Xb)
+    Y = torch.empty((m, n), dtype=torch.float32, device="cuda")
+
+    def call(st):
+        if noalloc:
+            sss.sss_gemm_noalloc(qt, X, Y, dev_status=st)
+        else:
+            sss.sss_gemm(qt, X, y=Y, dev_status=st)
+
+    status = _stalled(sss.TEST_STALL_GEMM, call)
+    assert status & sss.FLAG_TIMEOUT, status
+
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    Y.fill_(float("nan"))
+    call(st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    What = oracle.dequantize(codes, scales, mins, n, k, q, g, GRID)
+    Yref = oracle.matmul_f64(What, Xb)
+    assert rel_err_per_row(Y.cpu().numpy(), Yref).max() <= REL_TOL
+
+
+def test_stall_mask_off_by_default():
+    # the hook is process-wide: every test above clears it; a plain call here
+    # must see no timeout
+    n, k, q, g = 16, 4096, 2, 32
+    qt, (codes, scales, mins) = _packed(n, k, q, g, 25)
+    xb = x_bits(1, k, 8)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    y = sss.sss_gemv(qt, _x(xb), dev_status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    yref = oracle.gemv(codes, scales, mins, n, k, q, g, GRID, xb)
+    assert rel_err_per_row(y.cpu().numpy(), yref).max() <= REL_TOL
