@@ -1,8 +1,7 @@
-// gemv_common.cuh -- pieces of the batch-1 streaming GEMV (gemv_stream.cu):
-// bounded mbarrier waits, the fp16-subnormal code unpack feeding
-// mma.sync m16n8k16, and the staging of
-// the activation vector in mma order with the per-sub-chunk sums of the
-// Appendix B.3 row-sum term.
+// gemv_common.cuh -- pieces shared by the decode GEMV kernels
+// (gemv_stream.cu, gemv_batch.cu): bounded mbarrier waits, mma.sync
+// m16n8k16 wrappers, shared-memory loads, and the code-pair unpack of the
+// batched kernel (fields at bit 0, 2 or 4 of each fp16 half).
 #pragma once
 
 #include <stdint.h>
@@ -17,9 +16,6 @@ constexpr uint64_t kWaitNs = 1000000000ull;
 // fp16 pairs per 32-code sub-chunk: every width uses 16 (q=3 merges its two
 // bit planes into 3-bit fields before the mma)
 constexpr int NP = 16;
-// bytes of one sub-chunk's staged activations (16 pairs; no padding: the
-// 16-byte chunks are XOR-swizzled instead, see stage_x)
-constexpr int XPITCH = NP * 4;
 
 __device__ __forceinline__ uint32_t su32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -143,71 +139,6 @@ __device__ __forceinline__ uint32_t unpack_pair(const uint32_t* w, int p) {
       const int d = pos + 2 - e;
       const uint32_t hs = d >= 0 ? (hw << d) : (hw >> (-d));
       return lo | (hs & (0x00040004u << pos));
-    }
-  }
-}
-
-// Stage the bf16 activations x[0..32*nsc) in shared memory for the mma B
-// operand.  Sub-chunk i (32 elements) becomes NP fp16 pairs in unpack order,
-// each pre-divided by the power of two its code position carries; its four
-// 16-byte chunks c sit at xs + i*XPITCH + 16*(c ^ ((i >> 1) & 3)), a swizzle
-// under which the four sub-chunks one mma reads fall in distinct banks.
-// bias[i] = the sub-chunk's sum times 2^-24 (min-max grid) or times
-// -2^(q-1) * 2^-24 (symmetric grids).  Two threads share a sub-chunk (16
-// elements each); threads tid = 0..nthreads-1 (nthreads even) share the
-// work; the caller synchronises afterwards.
-template <int Q, bool ASYM>
-__device__ __forceinline__ void stage_x(const uint16_t* x, int nsc, uint32_t xs_a, float* bias,
-                                        int tid, int nthreads) {
-  constexpr int HALF = 1 << (Q - 1);
-  const int rounds = (2 * nsc + nthreads - 1) / nthreads;
-  for (int r = 0; r < rounds; ++r) {
-    const int t = tid + r * nthreads;
-    const bool valid = t < 2 * nsc;
-    const int i = t >> 1, hf = t & 1;
-    float xv[16];
-    if (valid) {
-      const uint4* src = reinterpret_cast<const uint4*>(x + static_cast<int64_t>(i) * 32 + 16 * hf);
-#pragma unroll
-      for (int c = 0; c < 2; ++c) {
-        const uint4 v = __ldg(src + c);
-        const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          xv[8 * c + 2 * e] = __uint_as_float(wv[e] << 16);
-          xv[8 * c + 2 * e + 1] = __uint_as_float(wv[e] & 0xFFFF0000u);
-        }
-      }
-    } else {
-#pragma unroll
-      for (int e = 0; e < 16; ++e) xv[e] = 0.f;
-    }
-    float sum = 0.f;
-#pragma unroll
-    for (int e = 0; e < 16; ++e) sum += xv[e];
-    sum += __shfl_xor_sync(0xffffffffu, sum, 1);
-    if (valid) {
-      uint32_t pr[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        // pair 8hf + j; both its elements lie in this half, at the same
-        // offsets from the half's start for either half
-        int ea, eb;
-        float mult;
-        pair_desc<Q>(j, ea, eb, mult);
-        __half2 hv = __floats2half2_rn(xv[ea] * mult, xv[eb] * mult);
-        pr[j] = *reinterpret_cast<uint32_t*>(&hv);
-      }
-      const uint32_t row = xs_a + static_cast<uint32_t>(i * XPITCH);
-      const int sw = (i >> 1) & 3;
-#pragma unroll
-      for (int c = 0; c < 2; ++c) {
-        const uint32_t dst = row + 16u * static_cast<uint32_t>((2 * hf + c) ^ sw);
-        asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(dst), "r"(pr[4 * c]),
-                     "r"(pr[4 * c + 1]), "r"(pr[4 * c + 2]), "r"(pr[4 * c + 3])
-                     : "memory");
-      }
-      if (hf == 0) bias[i] = ASYM ? sum * 0x1p-24f : -static_cast<float>(HALF) * 0x1p-24f * sum;
     }
   }
 }

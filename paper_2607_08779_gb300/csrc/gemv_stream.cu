@@ -2,11 +2,16 @@
 // packed q-bit codes (sm_103a), the streaming path of sss_gemv and
 // sss_gemv_multi.
 //
-// Same arithmetic as gemv.cu (Appendix B.3 expansion; codes unpacked as fp16
-// subnormals into mma.sync m16n8k16 with one B column per 32-code
-// sub-chunk; per-group scale and the row-sum term in fp32), organised for
-// streaming bandwidth:
+// Arithmetic (Appendix B.3 expansion): y = sum over groups of
+// s * (sum u*x - 2^(q-1) * sum x) for the symmetric grids, s * sum u*x +
+// m * sum x for the min-max grid, the integer part on the tensor cores:
+// codes are masked in place into fp16 operands (u * 2^pos * 2^-24, exact)
+// for mma.sync m16n8k16 with one B column per 32-code sub-chunk, and the
+// activations are staged as fp16 with a power of two per sub-chunk that
+// keeps them exact whatever their magnitude; scale, min and the row-sum
+// term are applied per group in fp32.
 //
+// Organisation, for streaming bandwidth:
 //  * persistent CTAs of 16 warps, one per SM, walking 16-row tiles of all
 //    jobs (several weight matrices sharing one activation vector, e.g. a
 //    fused q/k/v projection) round-robin;
@@ -44,6 +49,143 @@ constexpr int kThreads = kWarps * 32;
 constexpr int kMaxJobs = 4;
 using namespace gv;
 
+// ---------------------------------------------------------------------------
+// Code fields as fp16 operands.  An fp16 bit pattern below 2048 (exponent
+// field 0 or 1) has the value pattern * 2^-24, so a code masked in place at
+// bit position pos of a 16-bit half (its top bit at most bit 10) is the
+// operand u * 2^pos * 2^-24; the staged activation of that element carries
+// 2^-pos.  Pair p of a 32-code sub-chunk holds elements ea (low half) and
+// eb (high half):
+//   q=4: p = 4w + i: elements 8w+i and 8w+i+4 at pos 0 (i even) or 4 (i odd),
+//        nibble pairs 2 and 3 of each byte pair after one 8-bit shift;
+//   q=2, q=3: p = 8w + e: elements 16w+e and 16w+e+8, whose 2-bit low fields
+//        sit at bit 2e (e = 0..4) or, after one 10-bit shift, 2(e-5);
+//        q=3 ORs the element's high-plane bit in at pos + 2.
+// ---------------------------------------------------------------------------
+template <int Q>
+__device__ __forceinline__ void field_desc(int p, int& ea, int& eb, int& pos) {
+  if (Q == 4) {
+    const int w = p >> 2, i = p & 3;
+    ea = 8 * w + i;
+    eb = ea + 4;
+    pos = (i & 1) ? 4 : 0;
+  } else {
+    const int w = p >> 3, e = p & 7;
+    ea = 16 * w + e;
+    eb = ea + 8;
+    pos = e < 5 ? 2 * e : 2 * (e - 5);
+  }
+}
+
+// the high-plane bits of elements 16w .. 16w+15 (w = word of the sub-chunk)
+// spread to every other bit: element 16w+e at bit 2e (e < 8) and element
+// 16w+8+e at bit 16+2e
+__device__ __forceinline__ uint32_t spread_high(uint32_t hi_plane, int w) {
+  uint32_t x = __byte_perm(hi_plane, 0u, w ? 0x4342u : 0x4140u);
+  x = (x | (x << 4)) & 0x0F0F0F0Fu;
+  x = (x | (x << 2)) & 0x33333333u;
+  x = (x | (x << 1)) & 0x55555555u;
+  return x;
+}
+
+// Operand of pair p.  w[0..3] (q=4), w[0..1] (q=2) or w[0..1] + the high
+// plane w[2] (q=3) of one sub-chunk; hs[0..1] = spread_high of w[2] for q=3.
+template <int Q>
+__device__ __forceinline__ uint32_t field_pair(const uint32_t* w, const uint32_t* hs, int p) {
+  if constexpr (Q == 4) {
+    const uint32_t v = (p & 2) ? (w[p >> 2] >> 8) : w[p >> 2];
+    return v & ((p & 1) ? 0x00F000F0u : 0x000F000Fu);
+  } else {
+    const int wi = (p >> 3) & 1, e = p & 7;
+    const int pos = e < 5 ? 2 * e : 2 * (e - 5);
+    const uint32_t v = e < 5 ? w[wi] : (w[wi] >> 10);
+    const uint32_t lo = v & (0x00030003u << pos);
+    if constexpr (Q == 2) {
+      return lo;
+    } else {
+      // high bit of element e at 2e in hs; wanted at pos + 2
+      const uint32_t h = e < 5 ? (hs[wi] << 2) : (hs[wi] >> 8);
+      return lo | (h & (0x00040004u << pos));
+    }
+  }
+}
+
+// Stage the activations x[0 .. 32*nsc) for the mma B operand.  Sub-chunk i
+// (32 elements, 64 bytes at xs + 64 i) holds its 16 fp16 pairs in pair
+// order, element e as fl16(x_e * 2^(E_i - pos_e)): E_i is a power of two
+// chosen per sub-chunk so that its largest |x| lands in [2^14, 2^15), which
+// keeps every element exact in fp16 whatever the activations' magnitude.
+// sbf[i] = {b_i, f_i}: f_i = 2^(24 - E_i) undoes both scalings in the
+// epilogue, and b_i is the row-sum term of Appendix B.3 on the mma's scale:
+// sum(x) * 2^(E_i - 24), times -2^(q-1) for the symmetric grids.  Two
+// threads share a sub-chunk (16 elements each); threads tid = 0 ..
+// nthreads-1 (nthreads even) share the work; the caller synchronises.
+template <int Q, bool ASYM>
+__device__ __forceinline__ void stage_x(const uint16_t* x, int nsc, uint32_t xs_a, float2* sbf,
+                                        int tid, int nthreads) {
+  constexpr int HALF = 1 << (Q - 1);
+  const int rounds = (2 * nsc + nthreads - 1) / nthreads;
+  for (int r = 0; r < rounds; ++r) {
+    const int t = tid + r * nthreads;
+    const bool valid = t < 2 * nsc;
+    const int i = t >> 1, hf = t & 1;
+    float xv[16];
+    if (valid) {
+      const uint4* src = reinterpret_cast<const uint4*>(x + static_cast<int64_t>(i) * 32 + 16 * hf);
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        const uint4 v = __ldg(src + c);
+        const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          xv[8 * c + 2 * e] = __uint_as_float(wv[e] << 16);
+          xv[8 * c + 2 * e + 1] = __uint_as_float(wv[e] & 0xFFFF0000u);
+        }
+      }
+    } else {
+#pragma unroll
+      for (int e = 0; e < 16; ++e) xv[e] = 0.f;
+    }
+    float sum = 0.f, amax = 0.f;
+#pragma unroll
+    for (int e = 0; e < 16; ++e) {
+      sum += xv[e];
+      amax = fmaxf(amax, fabsf(xv[e]));
+    }
+    sum += __shfl_xor_sync(0xffffffffu, sum, 1);
+    amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 1));
+    // E = 14 - floor(log2 amax), kept in [-100, 100] (0 for a zero sub-chunk)
+    const int ex = static_cast<int>((__float_as_uint(amax) >> 23) & 0xFFu) - 127;
+    const int E = amax == 0.f ? 0 : max(-100, min(100, 14 - ex));
+    if (valid) {
+      uint32_t pr[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        // pair 8hf + j; both its elements lie in this half, at the same
+        // offsets from the half's start for either half
+        int ea, eb, pos;
+        field_desc<Q>(j, ea, eb, pos);
+        const float m = __int_as_float((127 + E - pos) << 23);  // 2^(E - pos)
+        __half2 hv = __floats2half2_rn(xv[ea] * m, xv[eb] * m);
+        pr[j] = *reinterpret_cast<uint32_t*>(&hv);
+      }
+      const uint32_t dst = xs_a + static_cast<uint32_t>(i * 64 + 32 * hf);
+      asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(dst), "r"(pr[0]), "r"(pr[1]),
+                   "r"(pr[2]), "r"(pr[3])
+                   : "memory");
+      asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(dst + 16u), "r"(pr[4]),
+                   "r"(pr[5]), "r"(pr[6]), "r"(pr[7])
+                   : "memory");
+      if (hf == 0) {
+        const float toE = __int_as_float((127 + E - 24) << 23);  // 2^(E - 24)
+        const float b = sum * toE;
+        sbf[i] = make_float2(ASYM ? sum : -static_cast<float>(HALF) * b,
+                             __int_as_float((127 + 24 - E) << 23));  // 2^(24 - E)
+      }
+    }
+  }
+}
+
 
 struct StreamJob {
   const uint8_t* codes;
@@ -80,9 +222,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   const int ngrp = kWarps >> lgkw;             // tiles in flight per CTA
 
   // ---- shared memory carve-up ----
-  unsigned char* xs = smem;                                                 // [nsc][XPITCH]
-  float* bias = reinterpret_cast<float*>(xs + static_cast<size_t>(nsc) * XPITCH);  // [nsc]
-  uint64_t* pready = reinterpret_cast<uint64_t*>(bias + ((nsc + 1) & ~1));  // [kWarps][2]
+  // staged activations [nsc][64 B] | two 64-byte zero blocks, the first 128
+  // bytes past a 128-aligned offset (the B operand of lanes that carry no
+  // data; see compute) | per-sub-chunk {b, f} | barriers | partials | flag
+  unsigned char* xs = smem;
+  const uint32_t zoff = (static_cast<uint32_t>(nsc) * 64u + 127u) & ~127u;
+  float2* sbf = reinterpret_cast<float2*>(xs + zoff + 128);              // [nsc]
+  uint64_t* pready = reinterpret_cast<uint64_t*>(sbf + nsc);              // [kWarps][2]
   uint64_t* pfree = pready + 2 * kWarps;                                   // [kWarps][2]
   float* part = reinterpret_cast<float*>(pfree + 2 * kWarps);              // [kWarps][2][R]
   volatile int* abort = reinterpret_cast<volatile int*>(part + 2 * kWarps * R);
@@ -101,6 +247,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
     *abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  if (threadIdx.x >= 32 && threadIdx.x < 64)
+    reinterpret_cast<uint32_t*>(xs + zoff)[threadIdx.x - 32] = 0u;  // the zero blocks
   // allow the next kernel in the stream to be scheduled as SMs free up
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
@@ -220,26 +368,26 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   asm volatile("griddepcontrol.wait;" ::: "memory");  // x is produced upstream
 
   // ---- stage the activations in mma order, and per-sub-chunk sums ----
-  stage_x<Q, ASYM>(a.x, nsc, su32(xs), bias, threadIdx.x, kThreads);
+  stage_x<Q, ASYM>(a.x, nsc, su32(xs), sbf, threadIdx.x, kThreads);
   __syncthreads();
 
   bool ok = true;
   float acc[2] = {0.f, 0.f};
-  // column gq of B carries the lane's sub-chunk 8u + gq in the mma of parity
-  // h only when it is the sub-chunk of this quad's own A rows (gq == 2tq + h);
-  // otherwise the lane reads zeros
+  // Column gq of B carries sub-chunk 8u + gq of the unit in the mmas of
+  // parity h = gq & 1, from the one lane of quad gq >> 1 whose own A rows
+  // hold that sub-chunk (gq == 2tq + h); every other lane supplies zeros by
+  // reading a zero block.  That leaves one data lane per quarter-warp, and
+  // the zero block of each parity sits 64 bytes (mod 128) away from the data
+  // lanes' banks, so the 16-byte loads are free of bank conflicts.
   const bool act0 = gq == 2 * tq, act1 = gq == 2 * tq + 1;
-  // swizzle of the staged activations of sub-chunk 8u + gq
-  const int xsw = (gq >> 1) & 3;
-  // shared-memory addresses (32-bit) of the lane's B data of the unit being
-  // computed and of the sums of its two columns' sub-chunks
-  const uint32_t xs_a = su32(xs), bias_a = su32(bias);
+  const uint32_t xs_a = su32(xs), sbf_a = su32(sbf);
+  const uint32_t z0 = xs_a + zoff + 64u, z1 = xs_a + zoff;  // zero blocks for h = 0, 1
   uint32_t xl = 0, bl = 0;
   int cleft = 0;
   int64_t ci = 0;
   auto start_tile = [&]() {
-    xl = xs_a + static_cast<uint32_t>((kw * 8 + gq) * XPITCH);
-    bl = bias_a + static_cast<uint32_t>((kw * 8 + 2 * tq) * 4);
+    xl = xs_a + static_cast<uint32_t>((kw * 8 + gq) * 64);
+    bl = sbf_a + static_cast<uint32_t>((kw * 8 + 2 * tq) * 8);
     cleft = upw;
   };
   start_tile();
@@ -249,26 +397,35 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
     float dh[2][4];
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      const bool act = h ? act1 : act0;
+      const uint32_t ba = h ? (act1 ? xl : z1) : (act0 ? xl : z0);
+      uint32_t hs0[2] = {0u, 0u}, hs1[2] = {0u, 0u};
+      if constexpr (Q == 3) {
+        hs0[0] = spread_high(rg.w[0][h][2], 0);
+        hs0[1] = spread_high(rg.w[0][h][2], 1);
+        hs1[0] = spread_high(rg.w[1][h][2], 0);
+        hs1[1] = spread_high(rg.w[1][h][2], 1);
+      }
 #pragma unroll
       for (int jm = 0; jm < NP / 2; jm += 2) {
-        uint4 bv = make_uint4(0u, 0u, 0u, 0u);
-        if (act) bv = lds128(xl + 16u * static_cast<uint32_t>((jm >> 1) ^ xsw));
+        const uint4 bv = lds128(ba + 8u * static_cast<uint32_t>(jm));
 #pragma unroll
         for (int jj = 0; jj < 2; ++jj) {
           const int p = 2 * (jm + jj);
+          const uint32_t a0 = field_pair<Q>(rg.w[0][h], hs0, p);
+          const uint32_t a1 = field_pair<Q>(rg.w[1][h], hs1, p);
+          const uint32_t a2 = field_pair<Q>(rg.w[0][h], hs0, p + 1);
+          const uint32_t a3 = field_pair<Q>(rg.w[1][h], hs1, p + 1);
           if (jm == 0 && jj == 0)
-            mma16816_z(dh[h], unpack_pair<Q>(rg.w[0][h], p), unpack_pair<Q>(rg.w[1][h], p),
-                       unpack_pair<Q>(rg.w[0][h], p + 1), unpack_pair<Q>(rg.w[1][h], p + 1),
-                       bv.x, bv.y);
+            mma16816_z(dh[h], a0, a1, a2, a3, bv.x, bv.y);
           else
-            mma16816(dh[h], unpack_pair<Q>(rg.w[0][h], p), unpack_pair<Q>(rg.w[1][h], p),
-                     unpack_pair<Q>(rg.w[0][h], p + 1), unpack_pair<Q>(rg.w[1][h], p + 1),
-                     jj ? bv.z : bv.x, jj ? bv.w : bv.y);
+            mma16816(dh[h], a0, a1, a2, a3, jj ? bv.z : bv.x, jj ? bv.w : bv.y);
         }
       }
     }
-    const float2 bb = lds64f(bl);
+    // {b, f} of the lane's sub-chunks 8u + 2tq and 8u + 2tq + 1
+    const uint4 bfv = lds128(bl);
+    const float b0 = __uint_as_float(bfv.x), f0 = __uint_as_float(bfv.y);
+    const float b1 = __uint_as_float(bfv.z), f1 = __uint_as_float(bfv.w);
 #pragma unroll
     for (int hh = 0; hh < 2; ++hh) {
       float s_0, s_1, m_0 = 0.f, m_1 = 0.f;
@@ -287,13 +444,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
       }
       const float d0 = dh[0][2 * hh], d1 = dh[1][2 * hh + 1];
       if constexpr (ASYM) {
-        acc[hh] += s_0 * d0 + m_0 * bb.x + s_1 * d1 + m_1 * bb.y;
+        acc[hh] += (s_0 * f0) * d0 + m_0 * b0 + (s_1 * f1) * d1 + m_1 * b1;
       } else {
-        acc[hh] += s_0 * (d0 + bb.x) + s_1 * (d1 + bb.y);
+        acc[hh] += (s_0 * f0) * (d0 + b0) + (s_1 * f1) * (d1 + b1);
       }
     }
-    xl += static_cast<uint32_t>(8 * XPITCH * KW);
-    bl += static_cast<uint32_t>(32 * KW);
+    xl += static_cast<uint32_t>(8 * 64 * KW);
+    bl += static_cast<uint32_t>(8 * 8 * KW);
   };
   auto tile_end = [&](int64_t i) {
     const int64_t t = tfirst + i * tstride;
@@ -315,7 +472,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
           const int64_t r = row0 + gq + 8 * hh;
-          if (r < jb.n) jb.y[r] = v[hh] * 0x1p24f;
+          if (r < jb.n) jb.y[r] = v[hh];
         }
       }
       return;
@@ -341,7 +498,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
         float sum = 0.f;
         for (int c = 0; c < KW; ++c) sum += pb[c * R + lane];
         const int64_t r = row0 + lane;
-        if (r < jb.n && ok) jb.y[r] = sum * 0x1p24f;
+        if (r < jb.n && ok) jb.y[r] = sum;
       }
       __syncwarp();
       if (lane == 0) bar_arrive(fre);
@@ -386,18 +543,17 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   if (*abort && threadIdx.x == 0 && a.status != nullptr) atomicOr(a.status, SSS_FLAG_TIMEOUT);
 }
 
-template <int Q, bool ASYM>
-size_t smem_bytes(int64_t k, int depth) {
+// activations (rounded up to 128) | zero blocks | {b, f} | 4*kWarps
+// barriers | partials | flag
+size_t smem_bytes(int64_t k) {
   const int64_t nsc = k / 32;
-  // activations | sums | 4*kWarps barriers | partials | flag
-  (void)depth;
-  return static_cast<size_t>(nsc) * XPITCH + 4 * ((nsc + 1) & ~int64_t{1}) +
-         8 * 4 * kWarps + 4 * 2 * kWarps * 16 + 16;
+  return static_cast<size_t>((nsc * 64 + 127) / 128 * 128 + 128 + 8 * nsc) + 8 * 4 * kWarps +
+         4 * 2 * kWarps * 16 + 16;
 }
 
 template <int Q, bool ASYM, int G, int D>
 cudaError_t launch_d(StreamArgs& a, int grid, bool pdl, cudaStream_t stream) {
-  const size_t smem = smem_bytes<Q, ASYM>(a.k, D);
+  const size_t smem = smem_bytes(a.k);
   auto kern = gemv_stream_kernel<Q, ASYM, G, D>;
   cudaError_t e = ensure_smem(kern, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
@@ -416,7 +572,7 @@ cudaError_t launch_d(StreamArgs& a, int grid, bool pdl, cudaStream_t stream) {
 
 template <int Q, bool ASYM, int G>
 cudaError_t launch_g(StreamArgs& a, int grid, bool pdl, cudaStream_t stream) {
-  if (smem_bytes<Q, ASYM>(a.k, 0) > 227 * 1024) return cudaErrorNotSupported;
+  if (smem_bytes(a.k) > 227 * 1024) return cudaErrorNotSupported;
   return launch_d<Q, ASYM, G, 2>(a, grid, pdl, stream);
 }
 
@@ -469,9 +625,7 @@ bool gemv_stream_eligible(const sss_qtensor_t& t, const uint16_t* x) {
   if (!al(t.codes, 16) || !al(t.scales, 4) || !al(x, 16)) return false;
   if (t.grid == SSS_GRID_ASYM && !al(t.mins, 4)) return false;
   // the staged activations must fit in shared memory
-  const int64_t nsc = t.k / 32;
-  const int64_t xbytes = nsc * (gv::XPITCH + 4);
-  return xbytes + 4096 <= 227 * 1024;
+  return smem_bytes(t.k) <= 227 * 1024;
 }
 
 cudaError_t launch_gemv_stream(const sss_qtensor_t* const* ts, float* const* ys, int count,

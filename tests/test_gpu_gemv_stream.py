@@ -110,3 +110,40 @@ def test_stream_ragged_jobs(g, grid):
     check_multi([1000, 33, 7, 250], 3072, 4, g, grid, 70 + g + grid)
     check_multi([517], 1024, 3, g, grid, 71 + g + grid)
     check_multi([96, 1], 2048, 2, g, grid, 72 + g + grid)
+
+
+def check_scaled_x(n, k, q, g, grid, seed, scale_of_chunk):
+    """The GEMV with activations whose 32-element sub-chunks are scaled by
+    scale_of_chunk(i) (powers of ten over many orders of magnitude, or all
+    small): bf16 values the fp16 mma operand cannot hold unscaled."""
+    qt, (codes, scales, mins) = make(n, k, q, g, grid, seed)
+    x = inputs.bf16_bits_to_f32(x_bits(1, k, seed + 3))[0].astype(np.float64)
+    x = x * np.repeat([scale_of_chunk(i) for i in range(k // 32)], 32)
+    xb = inputs.f32_to_bf16_bits(x.astype(np.float32)[None, :])
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    y = sss.sss_gemv_multi([qt], to_dev(xb[0].view(np.int16)).view(torch.bfloat16),
+                           dev_status=st)[0]
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    yref = oracle.gemv(codes, scales, mins, n, k, q, g, grid, xb)
+    err = rel_err_per_row(y.cpu().numpy()[None, :], yref)
+    assert err.max() <= REL_TOL, f"rel err {err.max():.3e}"
+    return float(err.max())
+
+
+@pytest.mark.parametrize("grid", GRIDS)
+@pytest.mark.parametrize("q", QS)
+@pytest.mark.parametrize("scale", [1e-4, 1e-6, 3e4])
+def test_stream_small_and_large_activations(q, grid, scale):
+    """Every element scaled alike: the result must not depend on where the
+    activations sit in the fp16 range."""
+    assert check_scaled_x(256, 2048, q, 32, grid, 80 + q, lambda i: scale) < 1e-4
+
+
+@pytest.mark.parametrize("q", QS)
+@pytest.mark.parametrize("g", [32, 128])
+def test_stream_activation_scale_varies_per_chunk(q, g):
+    """Sub-chunk magnitudes from 1e-8 to 1e4: the few large chunks dominate
+    the dot product, the small ones must not be lost or overflow."""
+    check_scaled_x(300, 4096, q, g, sss.GRID_SIGNED_SYM, 90 + q + g,
+                   lambda i: 10.0 ** ((i * 7) % 13 - 8))
