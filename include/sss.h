@@ -169,6 +169,11 @@ sss_status_t sss_gemv(const sss_qtensor_t* qt, const uint16_t* x_bf16,
 #define SSS_GEMV_WEIGHTS_READY 0x2u /* with SSS_GEMV_PDL: the packed weights are not written
                                        by the preceding work in the stream, so they may be
                                        streamed in before it completes                     */
+#define SSS_GEMV_ACT_Q8 0x4u        /* quantize x to Q8_0 on the fly (see
+                                       sss_quantize_act_q8) and multiply the packed
+                                       weights with the Q8_0 values: y_j[r] =
+                                       sum_blocks fl16(d) * sum_k w^_j[r][k] * q[k]; the
+                                       integer dot of codes and int8 values is exact */
 
 /*
  * sss_gemv_multi -- batch-1 decode GEMV of several packed matrices that
@@ -185,8 +190,9 @@ sss_status_t sss_gemv(const sss_qtensor_t* qt, const uint16_t* x_bf16,
  *   flags   [in]  SSS_GEMV_* bits.
  *   dev_status [out] nullable; SSS_FLAG_TIMEOUT if a bounded wait expired.
  * Shapes with k % 256 != 0 or k % (8*group) != 0, or unaligned buffers, run
- * as one sss_gemv per matrix (flags then have no effect).
- * Errors: SSS_E_ARG, SSS_E_ALIGN, SSS_E_CUDA.
+ * as one sss_gemv per matrix (flags then have no effect, and SSS_GEMV_ACT_Q8
+ * returns SSS_E_UNSUPPORTED).
+ * Errors: SSS_E_ARG, SSS_E_ALIGN, SSS_E_UNSUPPORTED, SSS_E_CUDA.
  */
 sss_status_t sss_gemv_multi(const sss_qtensor_t* const* qts, float* const* ys,
                             int32_t count, const uint16_t* x_bf16, uint32_t flags,
@@ -210,6 +216,93 @@ sss_status_t sss_gemv_multi(const sss_qtensor_t* const* qts, float* const* ys,
 sss_status_t sss_gemm(const sss_qtensor_t* qt, const uint16_t* x_bf16,
                       int64_t m, float* y, void* workspace, size_t ws_bytes,
                       uint32_t* dev_status, void* stream);
+
+/*
+ * sss_gemm_q8 -- sss_gemm on Q8_0 activations: each token's X is quantized
+ * per block of 32 (sss_quantize_act_q8) and the GEMM multiplies the packed
+ * weights with fl16(fl16(d) * q), the fp16 operand of the tensor cores (one
+ * rounding, <= 2^-11 relative).  This is the runtime pairing of few-bit
+ * weights with 8-bit activations the paper deploys (Sec. 5 "Composition with
+ * PTQ methods"; Appendix B.3 product).  Arguments, layouts, workspace and
+ * errors as sss_gemm; dev_status also receives the activation flags of
+ * sss_quantize_act_q8.
+ */
+sss_status_t sss_gemm_q8(const sss_qtensor_t* qt, const uint16_t* x_bf16,
+                         int64_t m, float* y, void* workspace, size_t ws_bytes,
+                         uint32_t* dev_status, void* stream);
+
+/*
+ * sss_quantize_act_q8 -- Q8_0 activations, the narrow-range 8-bit format the
+ * paper pairs with its weight formats (Sec. 5 "Composition with PTQ
+ * methods"; Appendix C "Algorithm details"): per block of 32 consecutive
+ * values of a row, M = max |x|, d = fl32(M / 127), q = clip(RNE(x / d) of
+ * the exact quotient, -127, 127), stored scale fl16(d).  A zero block gives
+ * q = 0, d = +0; a block with NaN/Inf gives q = 0, d = +0 and
+ * SSS_FLAG_NONFINITE; an fp16 overflow of d raises SSS_FLAG_RANGE.
+ *   x_bf16 [in]  device bf16 [rows][k], 16-byte aligned; k % 32 == 0.
+ *   q      [out] device int8 [rows][k], 8-byte aligned.
+ *   d      [out] device fp16 [rows][k/32].
+ * Errors: SSS_E_ARG, SSS_E_ALIGN, SSS_E_CUDA.
+ */
+sss_status_t sss_quantize_act_q8(const uint16_t* x_bf16, int64_t rows, int64_t k,
+                                 int8_t* q, uint16_t* d, uint32_t* dev_status,
+                                 void* stream);
+
+/*
+ * Normalized Hadamard rotation of the weights before quantization: the
+ * mergeable rotations of the paper's PTQ pipeline (Sec. 5 "Composition with
+ * PTQ methods"; Appendix C, the rotation graph), folded into the weights so
+ * that the grids are computed on the rotated weights and the runtime path
+ * is unchanged.  The transform of a block of b values (b a power of two,
+ * 2 <= b <= 8192) is the normalized Walsh-Hadamard transform H_b/sqrt(b)
+ * (Sylvester order) computed as the in-place fast transform in IEEE fp32:
+ * strides h = 1, 2, ..., b/2, butterflies (a, c) -> (a + c, a - c), then
+ * every value times the fp32 nearest to 1/sqrt(b).  H_b/sqrt(b) is
+ * symmetric and orthogonal: W x = (W R)(R x) for R = I (x) H_b/sqrt(b).
+ */
+#define SSS_ROTATE_INPUT 0  /* W <- W R: every block of b consecutive values of a row (b | k) */
+#define SSS_ROTATE_OUTPUT 1 /* W <- R W: every block of b consecutive rows, per column
+                               (b | n, and k a multiple of 8192/b)                          */
+
+/*
+ * sss_hadamard -- rotate the fp32 matrix w [n][k] into out [n][k] (out may
+ * equal w).  Both 16-byte aligned.
+ * Errors: SSS_E_ARG (block, side or shape), SSS_E_ALIGN, SSS_E_CUDA.
+ */
+sss_status_t sss_hadamard(const float* w, float* out, int64_t n, int64_t k,
+                          int32_t block, int32_t side, void* stream);
+
+/*
+ * sss_quantize_rotated -- sss_quantize of the input-side rotation of w:
+ * bit for bit sss_hadamard(w, tmp, n, k, block, SSS_ROTATE_INPUT) followed
+ * by sss_quantize(tmp, out, ...), in one pass that never writes the rotated
+ * fp32 weights (block | k).  Arguments and errors as sss_quantize.
+ */
+sss_status_t sss_quantize_rotated(const float* w, int32_t block, const sss_qtensor_t* out,
+                                  uint8_t* clip_counts, uint32_t* dev_status,
+                                  void* stream);
+
+/*
+ * sss_sign_diagnostics -- the cardinality margin and the realised l2 gain of
+ * the signed absmax sign rule on every group (Sec. 4, rem:cardinality-margin
+ * and fig:theory-diagnostics), on any fp32 weights: for the sign gamma* of
+ * eq:sign_rule and the clipped sets of def:clipped-set,
+ *   margin m = |C_-gamma*| - |C_gamma*|            (in -group .. group)
+ *   gain   g = ||w - Q_-gamma*(w)||^2 - ||w - Q_gamma*(w)||^2
+ * with the weights each sign's stored fp16 scale dequantises to.  g is
+ * exact (fp64).  Groups with NaN/Inf are skipped and raise
+ * SSS_FLAG_NONFINITE; all-zero groups count as m = 0, g = 0.
+ *   w      [in]  device fp32 [n][k], 16-byte aligned; k % group == 0.
+ *   q      [in]  2, 3 or 4;  group 32, 64 or 128.
+ *   margin [out] nullable device int16 [n][k/group].
+ *   gain   [out] nullable device fp64 [n][k/group].
+ *   hist   [in,out] nullable device uint64 [2*group+1][3], ADDED to: row
+ *                m + group, column 0 (g < 0), 1 (g == 0) or 2 (g > 0).
+ * Errors: SSS_E_ARG, SSS_E_ALIGN, SSS_E_CUDA.
+ */
+sss_status_t sss_sign_diagnostics(const float* w, int64_t n, int64_t k, int32_t q,
+                                  int32_t group, int16_t* margin, double* gain,
+                                  uint64_t* hist, uint32_t* dev_status, void* stream);
 
 #define SSS_OP_GEMV 0
 #define SSS_OP_GEMM 1

@@ -553,13 +553,18 @@ cudaError_t gemm_grid(const sss_qtensor_t& t, const __half* x16, int64_t m, floa
 size_t gemm_workspace_bytes(const sss_qtensor_t& t, int64_t m) { return x16_bytes(m, t.k); }
 
 cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m, float* y,
-                        void* workspace, uint32_t* status, cudaStream_t stream) {
+                        void* workspace, uint32_t* status, cudaStream_t stream, bool act_q8) {
   __half* x16 = static_cast<__half*>(workspace);
-  const int64_t nvec = m * t.k / 8;
-  const int grid = static_cast<int>(std::min<int64_t>((nvec + 255) / 256,
-                                                      static_cast<int64_t>(device_sm_count()) * 8));
-  bf16_to_f16_kernel<<<std::max(grid, 1), 256, 0, stream>>>(x, x16, nvec);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e;
+  if (act_q8) {
+    e = launch_act_q8_f16(x, m, t.k, x16, status, stream);
+  } else {
+    const int64_t nvec = m * t.k / 8;
+    const int grid = static_cast<int>(std::min<int64_t>((nvec + 255) / 256,
+                                                        static_cast<int64_t>(device_sm_count()) * 8));
+    bf16_to_f16_kernel<<<std::max(grid, 1), 256, 0, stream>>>(x, x16, nvec);
+    e = cudaGetLastError();
+  }
   if (e != cudaSuccess) return e;
   switch (t.q) {
     case 2: return gemm_grid<2>(t, x16, m, y, status, stream);

@@ -39,6 +39,7 @@
 
 #include <algorithm>
 
+#include "act_q8.cuh"
 #include "gemv_common.cuh"
 
 namespace sss {
@@ -120,9 +121,17 @@ __device__ __forceinline__ uint32_t field_pair(const uint32_t* w, const uint32_t
 // sum(x) * 2^(E_i - 24), times -2^(q-1) for the symmetric grids.  Two
 // threads share a sub-chunk (16 elements each); threads tid = 0 ..
 // nthreads-1 (nthreads even) share the work; the caller synchronises.
+//
+// With act_q8 the activations are first quantized to Q8_0 (act_q8.cuh; a
+// sub-chunk is one Q8_0 block): the staged operand is the int8 code q
+// (times 2^-pos, exact in fp16), f_i = fl16(d_i) * 2^24 and the row-sum
+// term uses sum(q), so the mma's integer dot sum(u*q) is exact and the
+// block scale meets the group scale in fp32 (the Appendix B.3 product on
+// Q8_0 activations).  Non-finite or fp16-overflowing blocks set the status
+// bits as sss_quantize_act_q8 does.
 template <int Q, bool ASYM>
 __device__ __forceinline__ void stage_x(const uint16_t* x, int nsc, uint32_t xs_a, float2* sbf,
-                                        int tid, int nthreads) {
+                                        int tid, int nthreads, bool act_q8, uint32_t* status) {
   constexpr int HALF = 1 << (Q - 1);
   const int rounds = (2 * nsc + nthreads - 1) / nthreads;
   for (int r = 0; r < rounds; ++r) {
@@ -156,7 +165,30 @@ __device__ __forceinline__ void stage_x(const uint16_t* x, int nsc, uint32_t xs_
     amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 1));
     // E = 14 - floor(log2 amax), kept in [-100, 100] (0 for a zero sub-chunk)
     const int ex = static_cast<int>((__float_as_uint(amax) >> 23) & 0xFFu) - 127;
-    const int E = amax == 0.f ? 0 : max(-100, min(100, 14 - ex));
+    int E = amax == 0.f ? 0 : max(-100, min(100, 14 - ex));
+    float fq = 0.f;  // Q8_0: fl16(d) * 2^24
+    if (act_q8) {
+      unsigned bad = 0;
+#pragma unroll
+      for (int e = 0; e < 16; ++e) bad |= is_nonfinite(xv[e]);
+      bad |= __shfl_xor_sync(0xffffffffu, bad, 1);
+      unsigned flags = 0;
+      uint16_t d16;
+      const float d = q8_scale(amax, bad != 0, &d16, &flags);
+      const float r = d != 0.f ? __frcp_rn(d) : 0.f;
+      int qs = 0;
+#pragma unroll
+      for (int e = 0; e < 16; ++e) {
+        const int qv = d != 0.f ? q8_code(xv[e], d, r) : 0;
+        qs += qv;
+        xv[e] = static_cast<float>(qv);
+      }
+      qs += __shfl_xor_sync(0xffffffffu, qs, 1);
+      sum = static_cast<float>(qs);  // exact: |sum q| <= 32 * 127
+      E = 0;
+      fq = __half2float(__ushort_as_half(d16)) * 0x1p24f;
+      if (valid && hf == 0 && flags != 0u && status != nullptr) atomicOr(status, flags);
+    }
     if (valid) {
       uint32_t pr[8];
 #pragma unroll
@@ -179,8 +211,10 @@ __device__ __forceinline__ void stage_x(const uint16_t* x, int nsc, uint32_t xs_
       if (hf == 0) {
         const float toE = __int_as_float((127 + E - 24) << 23);  // 2^(E - 24)
         const float b = sum * toE;
-        sbf[i] = make_float2(ASYM ? sum : -static_cast<float>(HALF) * b,
-                             __int_as_float((127 + 24 - E) << 23));  // 2^(24 - E)
+        const float f = act_q8 ? fq : __int_as_float((127 + 24 - E) << 23);  // 2^(24 - E)
+        // min-max grid: b is the block's sum of activation values
+        const float bsum = act_q8 ? fq * b : sum;
+        sbf[i] = make_float2(ASYM ? bsum : -static_cast<float>(HALF) * b, f);
       }
     }
   }
@@ -204,6 +238,7 @@ struct StreamArgs {
   int64_t ntiles;
   int lgkw;            // log2(warps per tile)
   int early_weights;   // prefetch weights before the grid-dependency wait
+  int act_q8;          // quantize the activations to Q8_0 while staging them
   int stall;           // test hook: one partial of the first tile is never announced
   uint32_t* status;
 };
@@ -368,7 +403,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   asm volatile("griddepcontrol.wait;" ::: "memory");  // x is produced upstream
 
   // ---- stage the activations in mma order, and per-sub-chunk sums ----
-  stage_x<Q, ASYM>(a.x, nsc, su32(xs), sbf, threadIdx.x, kThreads);
+  stage_x<Q, ASYM>(a.x, nsc, su32(xs), sbf, threadIdx.x, kThreads, a.act_q8 != 0, a.status);
   __syncthreads();
 
   bool ok = true;
@@ -638,6 +673,7 @@ cudaError_t launch_gemv_stream(const sss_qtensor_t* const* ts, float* const* ys,
   a.x = x;
   a.k = ts[0]->k;
   a.early_weights = (flags & SSS_GEMV_WEIGHTS_READY) ? 1 : 0;
+  a.act_q8 = (flags & SSS_GEMV_ACT_Q8) ? 1 : 0;
   a.stall = (test_stall_mask() & SSS_TEST_STALL_GEMV) ? 1 : 0;
   a.status = status;
   for (int j = 0; j < count; ++j) {

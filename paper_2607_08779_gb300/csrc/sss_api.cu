@@ -218,7 +218,7 @@ sss_status_t sss_gemv_multi(const sss_qtensor_t* const* qts, float* const* ys, i
                             const uint16_t* x_bf16, uint32_t flags, uint32_t* dev_status,
                             void* stream) {
   if (qts == nullptr || ys == nullptr || count < 1 || count > 4) return SSS_E_ARG;
-  if ((flags & ~(SSS_GEMV_PDL | SSS_GEMV_WEIGHTS_READY)) != 0) return SSS_E_ARG;
+  if ((flags & ~(SSS_GEMV_PDL | SSS_GEMV_WEIGHTS_READY | SSS_GEMV_ACT_Q8)) != 0) return SSS_E_ARG;
   bool stream_ok = true;
   for (int j = 0; j < count; ++j) {
     sss_status_t st = check_tensor(qts[j]);
@@ -237,6 +237,8 @@ sss_status_t sss_gemv_multi(const sss_qtensor_t* const* qts, float* const* ys, i
     return finish("sss_gemv_multi", launch_gemv_stream(qts, ys, count, x_bf16, flags, dev_status,
                                                        static_cast<cudaStream_t>(stream)));
   }
+  // the general kernels take bf16 activations only
+  if (flags & SSS_GEMV_ACT_Q8) return SSS_E_UNSUPPORTED;
   for (int j = 0; j < count; ++j) {
     sss_status_t st = sss_gemv(qts[j], x_bf16, 1, ys[j], nullptr, 0, dev_status, stream);
     if (st != SSS_OK) return st;
@@ -244,9 +246,10 @@ sss_status_t sss_gemv_multi(const sss_qtensor_t* const* qts, float* const* ys, i
   return SSS_OK;
 }
 
-sss_status_t sss_gemm(const sss_qtensor_t* qt, const uint16_t* x_bf16, int64_t m,
-                      float* y, void* workspace, size_t ws_bytes,
-                      uint32_t* dev_status, void* stream) {
+namespace {
+sss_status_t gemm_common(const char* name, const sss_qtensor_t* qt, const uint16_t* x_bf16,
+                         int64_t m, float* y, void* workspace, size_t ws_bytes,
+                         uint32_t* dev_status, void* stream, bool act_q8) {
   sss_status_t st = check_tensor(qt);
   if (st != SSS_OK) return st;
   if (m < 0 || m > kMaxTokens) return SSS_E_ARG;
@@ -262,12 +265,88 @@ sss_status_t sss_gemm(const sss_qtensor_t* qt, const uint16_t* x_bf16, int64_t m
   if (need > 0 && (workspace == nullptr || ws_bytes < need)) return SSS_E_WORKSPACE;
   if (workspace != nullptr && !aligned(workspace, 16)) return SSS_E_ALIGN;
   if (qt->k == 0) {
-    return finish("sss_gemm",
-                  cudaMemsetAsync(y, 0, sizeof(float) * static_cast<size_t>(m) * qt->n,
-                                  static_cast<cudaStream_t>(stream)));
-  }
-  return finish("sss_gemm", launch_gemm(*qt, x_bf16, m, y, workspace, dev_status,
+    return finish(name, cudaMemsetAsync(y, 0, sizeof(float) * static_cast<size_t>(m) * qt->n,
                                         static_cast<cudaStream_t>(stream)));
+  }
+  return finish(name, launch_gemm(*qt, x_bf16, m, y, workspace, dev_status,
+                                  static_cast<cudaStream_t>(stream), act_q8));
+}
+}  // namespace
+
+sss_status_t sss_gemm(const sss_qtensor_t* qt, const uint16_t* x_bf16, int64_t m,
+                      float* y, void* workspace, size_t ws_bytes,
+                      uint32_t* dev_status, void* stream) {
+  return gemm_common("sss_gemm", qt, x_bf16, m, y, workspace, ws_bytes, dev_status, stream,
+                     false);
+}
+
+sss_status_t sss_gemm_q8(const sss_qtensor_t* qt, const uint16_t* x_bf16, int64_t m,
+                         float* y, void* workspace, size_t ws_bytes,
+                         uint32_t* dev_status, void* stream) {
+  if (qt != nullptr && qt->k % 32 != 0) return SSS_E_ARG;
+  return gemm_common("sss_gemm_q8", qt, x_bf16, m, y, workspace, ws_bytes, dev_status, stream,
+                     true);
+}
+
+namespace {
+bool pow2_block(int64_t b) { return b >= 2 && b <= 8192 && (b & (b - 1)) == 0; }
+}  // namespace
+
+sss_status_t sss_hadamard(const float* w, float* out, int64_t n, int64_t k, int32_t block,
+                          int32_t side, void* stream) {
+  if (n < 0 || k < 0 || n > kMaxDim || k > kMaxDim || !pow2_block(block)) return SSS_E_ARG;
+  if (side != SSS_ROTATE_INPUT && side != SSS_ROTATE_OUTPUT) return SSS_E_ARG;
+  if (side == SSS_ROTATE_INPUT && k % block != 0) return SSS_E_ARG;
+  if (side == SSS_ROTATE_OUTPUT && (n % block != 0 || k % (8192 / block) != 0)) return SSS_E_ARG;
+  if (n == 0 || k == 0) return SSS_OK;
+  if (w == nullptr || out == nullptr) return SSS_E_ARG;
+  if (!aligned(w, 16) || !aligned(out, 16)) return SSS_E_ALIGN;
+  return finish("sss_hadamard", launch_hadamard(w, out, n, k, block, side,
+                                                static_cast<cudaStream_t>(stream)));
+}
+
+sss_status_t sss_quantize_rotated(const float* w, int32_t block, const sss_qtensor_t* out,
+                                  uint8_t* clip_counts, uint32_t* dev_status, void* stream) {
+  sss_status_t st = check_tensor(out);
+  if (st != SSS_OK) return st;
+  if (!pow2_block(block) || out->k % block != 0) return SSS_E_ARG;
+  if (out->n == 0 || out->k == 0) return SSS_OK;
+  if (w == nullptr) return SSS_E_ARG;
+  if (!aligned(w, 16) || !aligned(out->codes, 16) || !aligned(out->scales, 2) ||
+      (out->mins && !aligned(out->mins, 2)) || (dev_status && !aligned(dev_status, 4)))
+    return SSS_E_ALIGN;
+  return finish("sss_quantize_rotated",
+                launch_quantize_rotated(w, block, *out, clip_counts, dev_status,
+                                        static_cast<cudaStream_t>(stream)));
+}
+
+sss_status_t sss_sign_diagnostics(const float* w, int64_t n, int64_t k, int32_t q,
+                                  int32_t group, int16_t* margin, double* gain,
+                                  uint64_t* hist, uint32_t* dev_status, void* stream) {
+  if (n < 0 || k < 0 || n > kMaxDim || k > kMaxDim) return SSS_E_ARG;
+  if (q < 2 || q > 4) return SSS_E_ARG;
+  if (group != 32 && group != 64 && group != 128) return SSS_E_ARG;
+  if (k % group != 0) return SSS_E_ARG;
+  if (n == 0 || k == 0) return SSS_OK;
+  if (w == nullptr) return SSS_E_ARG;
+  if (!aligned(w, 16) || (margin && !aligned(margin, 2)) || (gain && !aligned(gain, 8)) ||
+      (hist && !aligned(hist, 8)) || (dev_status && !aligned(dev_status, 4)))
+    return SSS_E_ALIGN;
+  return finish("sss_sign_diagnostics",
+                launch_sign_diagnostics(w, n, k, q, group, margin, gain,
+                                        reinterpret_cast<unsigned long long*>(hist), dev_status,
+                                        static_cast<cudaStream_t>(stream)));
+}
+
+sss_status_t sss_quantize_act_q8(const uint16_t* x_bf16, int64_t rows, int64_t k, int8_t* q,
+                                 uint16_t* d, uint32_t* dev_status, void* stream) {
+  if (rows < 0 || k < 0 || rows > kMaxDim || k > kMaxDim || k % 32 != 0) return SSS_E_ARG;
+  if (rows == 0 || k == 0) return SSS_OK;
+  if (x_bf16 == nullptr || q == nullptr || d == nullptr) return SSS_E_ARG;
+  if (!aligned(x_bf16, 16) || !aligned(q, 8) || !aligned(d, 2)) return SSS_E_ALIGN;
+  if (dev_status && !aligned(dev_status, 4)) return SSS_E_ALIGN;
+  return finish("sss_quantize_act_q8",
+                launch_act_q8(x_bf16, rows, k, q, d, dev_status, static_cast<cudaStream_t>(stream)));
 }
 
 }  // extern "C"

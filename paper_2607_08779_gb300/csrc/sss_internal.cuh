@@ -46,7 +46,21 @@ cudaError_t launch_gemv_batch(const sss_qtensor_t& t, const uint16_t* x, int bat
 size_t gemm_workspace_bytes(const sss_qtensor_t& t, int64_t m);
 cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m,
                         float* y, void* workspace, uint32_t* status,
-                        cudaStream_t stream);
+                        cudaStream_t stream, bool act_q8 = false);
+
+cudaError_t launch_act_q8(const uint16_t* x, int64_t rows, int64_t k, int8_t* q, uint16_t* d,
+                          uint32_t* status, cudaStream_t stream);
+cudaError_t launch_act_q8_f16(const uint16_t* x, int64_t rows, int64_t k, __half* out,
+                              uint32_t* status, cudaStream_t stream);
+
+cudaError_t launch_hadamard(const float* w, float* out, int64_t n, int64_t k, int b, int side,
+                            cudaStream_t stream);
+cudaError_t launch_quantize_rotated(const float* w, int b, const sss_qtensor_t& t, uint8_t* clip,
+                                    uint32_t* status, cudaStream_t stream);
+
+cudaError_t launch_sign_diagnostics(const float* w, int64_t n, int64_t k, int q, int g,
+                                    int16_t* margin, double* gain, unsigned long long* hist,
+                                    uint32_t* status, cudaStream_t stream);
 
 // The kernel families whose next launches skip one barrier arrive
 // (sss_test_set_stall; 0 in normal use).

@@ -32,10 +32,15 @@ STATUS_NAMES = {0: "SSS_OK", 1: "SSS_E_ARG", 2: "SSS_E_UNSUPPORTED", 3: "SSS_E_A
 
 EXPORTS = ("sss_codes_bytes", "sss_status_string", "sss_last_error", "sss_quantize",
            "sss_dequantize", "sss_gemv", "sss_gemv_multi", "sss_gemm", "sss_workspace_bytes",
-           "sss_gemm_noalloc", "sss_gemm_noalloc_max_scratch_bytes", "sss_test_set_stall")
+           "sss_gemm_noalloc", "sss_gemm_noalloc_max_scratch_bytes", "sss_test_set_stall",
+           "sss_gemm_q8", "sss_quantize_act_q8", "sss_sign_diagnostics", "sss_hadamard",
+           "sss_quantize_rotated")
 
 GEMV_PDL = 0x1
 GEMV_WEIGHTS_READY = 0x2
+GEMV_ACT_Q8 = 0x4
+
+ROTATE_INPUT, ROTATE_OUTPUT = 0, 1
 
 TEST_STALL_GEMV = 0x1
 TEST_STALL_GEMV_BATCH = 0x2
@@ -108,6 +113,16 @@ def load(build_if_needed: bool = True):
         L.sss_gemm_noalloc.restype = i32
         L.sss_gemm_noalloc_max_scratch_bytes.argtypes = []
         L.sss_gemm_noalloc_max_scratch_bytes.restype = sz
+        L.sss_gemm_q8.argtypes = [P, vp, i64, vp, vp, sz, vp, vp]
+        L.sss_gemm_q8.restype = i32
+        L.sss_quantize_act_q8.argtypes = [vp, i64, i64, vp, vp, vp, vp]
+        L.sss_quantize_act_q8.restype = i32
+        L.sss_sign_diagnostics.argtypes = [vp, i64, i64, i32, i32, vp, vp, vp, vp, vp]
+        L.sss_sign_diagnostics.restype = i32
+        L.sss_hadamard.argtypes = [vp, vp, i64, i64, i32, i32, vp]
+        L.sss_hadamard.restype = i32
+        L.sss_quantize_rotated.argtypes = [vp, i32, P, vp, vp, vp]
+        L.sss_quantize_rotated.restype = i32
         L.sss_test_set_stall.argtypes = [ctypes.c_uint32]
         L.sss_test_set_stall.restype = None
         _lib = L
@@ -311,19 +326,18 @@ def sss_gemv_multi(qts, x, ys=None, flags: int = 0, dev_status=None, stream=None
     return ys
 
 
-def sss_gemm(qt: QTensor, x, y=None, workspace=None, dev_status=None, stream=None):
-    """Y [m, n] fp32 = X [m, k] (bf16) @ dequant(qt)^T on the tensor cores."""
+def _gemm(fn: str, qt: QTensor, x, y, workspace, dev_status, stream):
     import torch
 
     m = x.shape[0]
-    _need("sss_gemm", "x", x, torch.bfloat16, m * qt.k)
+    _need(fn, "x", x, torch.bfloat16, m * qt.k)
     if y is None:
         y = torch.empty((m, qt.n), dtype=torch.float32, device=x.device)
-    _need("sss_gemm", "y", y, torch.float32, m * qt.n)
-    _need_qtensor("sss_gemm", qt)
-    _need("sss_gemm", "workspace", workspace, torch.uint8, optional=True)
-    _need_status("sss_gemm", dev_status)
-    _on_device("sss_gemm", x=x, y=y, codes=qt.codes, scales=qt.scales, mins=qt.mins,
+    _need(fn, "y", y, torch.float32, m * qt.n)
+    _need_qtensor(fn, qt)
+    _need(fn, "workspace", workspace, torch.uint8, optional=True)
+    _need_status(fn, dev_status)
+    _on_device(fn, x=x, y=y, codes=qt.codes, scales=qt.scales, mins=qt.mins,
                workspace=workspace, dev_status=dev_status)
     d = qt.desc()
     if workspace is None:
@@ -331,10 +345,41 @@ def sss_gemm(qt: QTensor, x, y=None, workspace=None, dev_status=None, stream=Non
         if need > 0:
             workspace = torch.empty(need, dtype=torch.uint8, device=x.device)
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
-    st = load().sss_gemm(ctypes.byref(d), _ptr(x), m, _ptr(y), _ptr(workspace), ws_bytes,
-                         _ptr(dev_status), _stream(stream))
-    _check("sss_gemm", st)
+    st = getattr(load(), fn)(ctypes.byref(d), _ptr(x), m, _ptr(y), _ptr(workspace), ws_bytes,
+                             _ptr(dev_status), _stream(stream))
+    _check(fn, st)
     return y
+
+
+def sss_gemm(qt: QTensor, x, y=None, workspace=None, dev_status=None, stream=None):
+    """Y [m, n] fp32 = X [m, k] (bf16) @ dequant(qt)^T on the tensor cores."""
+    return _gemm("sss_gemm", qt, x, y, workspace, dev_status, stream)
+
+
+def sss_gemm_q8(qt: QTensor, x, y=None, workspace=None, dev_status=None, stream=None):
+    """sss_gemm with X quantized to Q8_0 (per token, per block of 32) first."""
+    return _gemm("sss_gemm_q8", qt, x, y, workspace, dev_status, stream)
+
+
+def sss_quantize_act_q8(x, q=None, d=None, dev_status=None, stream=None):
+    """Q8_0 activations of bf16 x [rows, k]: int8 codes [rows, k] and fp16
+    block scales [rows, k/32] (returned as int16 bit patterns)."""
+    import torch
+
+    rows, k = x.shape
+    _need("sss_quantize_act_q8", "x", x, torch.bfloat16, rows * k)
+    if q is None:
+        q = torch.empty((rows, k), dtype=torch.int8, device=x.device)
+    if d is None:
+        d = torch.empty((rows, k // 32), dtype=torch.int16, device=x.device)
+    _need("sss_quantize_act_q8", "q", q, torch.int8, rows * k)
+    _need("sss_quantize_act_q8", "d", d, torch.int16, rows * (k // 32))
+    _need_status("sss_quantize_act_q8", dev_status)
+    _on_device("sss_quantize_act_q8", x=x, q=q, d=d, dev_status=dev_status)
+    st = load().sss_quantize_act_q8(_ptr(x), rows, k, _ptr(q), _ptr(d), _ptr(dev_status),
+                                    _stream(stream))
+    _check("sss_quantize_act_q8", st)
+    return q, d
 
 
 def sss_gemm_noalloc(qt: QTensor, x, y, dev_status=None, stream=None):
@@ -365,3 +410,71 @@ def sss_test_set_stall(mask: int) -> None:
     launches): later launches of the named kernels leave one barrier one
     arrive short, so a wait runs out and the kernel raises FLAG_TIMEOUT."""
     load().sss_test_set_stall(int(mask))
+
+
+def sss_sign_diagnostics(w, q: int, group: int, margin=None, gain=None, hist=None,
+                         dev_status=None, stream=None):
+    """Per-group cardinality margin (int16 [n, k/group]) and exact l2 gain
+    (float64 [n, k/group]) of the signed absmax sign rule, and their
+    histogram (int64 [2*group+1, 3], added to: row m + group, column g<0 /
+    g==0 / g>0).  Returns (margin, gain, hist)."""
+    import torch
+
+    n, k = w.shape
+    fn = "sss_sign_diagnostics"
+    _need(fn, "w", w, torch.float32, n * k)
+    ng = n * (k // group) if group > 0 else 0
+    if margin is None:
+        margin = torch.empty((n, k // group), dtype=torch.int16, device=w.device)
+    if gain is None:
+        gain = torch.empty((n, k // group), dtype=torch.float64, device=w.device)
+    if hist is None:
+        hist = torch.zeros((2 * group + 1, 3), dtype=torch.int64, device=w.device)
+    _need(fn, "margin", margin, torch.int16, ng)
+    _need(fn, "gain", gain, torch.float64, ng)
+    _need(fn, "hist", hist, torch.int64, (2 * group + 1) * 3)
+    _need_status(fn, dev_status)
+    _on_device(fn, w=w, margin=margin, gain=gain, hist=hist, dev_status=dev_status)
+    st = load().sss_sign_diagnostics(_ptr(w), n, k, q, group, _ptr(margin), _ptr(gain),
+                                     _ptr(hist), _ptr(dev_status), _stream(stream))
+    _check(fn, st)
+    return margin, gain, hist
+
+
+def sss_hadamard(w, block: int, side: int = ROTATE_INPUT, out=None, stream=None):
+    """The normalized Hadamard rotation of fp32 w [n, k] (block b, input or
+    output side) into out (new tensor if None; may be w itself)."""
+    import torch
+
+    n, k = w.shape
+    _need("sss_hadamard", "w", w, torch.float32, n * k)
+    if out is None:
+        out = torch.empty_like(w)
+    _need("sss_hadamard", "out", out, torch.float32, n * k)
+    _on_device("sss_hadamard", w=w, out=out)
+    st = load().sss_hadamard(_ptr(w), _ptr(out), n, k, block, side, _stream(stream))
+    _check("sss_hadamard", st)
+    return out
+
+
+def sss_quantize_rotated(w, block: int, q: int, group: int, grid: int,
+                         out: Optional["QTensor"] = None, clip_counts=None, dev_status=None,
+                         stream=None) -> "QTensor":
+    """sss_quantize of the input-side Hadamard rotation of w (block b), fused."""
+    import torch
+
+    n, k = w.shape
+    fn = "sss_quantize_rotated"
+    _need(fn, "w", w, torch.float32, n * k)
+    if out is None:
+        out = empty_qtensor(n, k, q, group, grid, device=w.device)
+    _need_qtensor(fn, out)
+    _need(fn, "clip_counts", clip_counts, torch.uint8, n * (k // group) * 2, optional=True)
+    _need_status(fn, dev_status)
+    _on_device(fn, w=w, codes=out.codes, scales=out.scales, mins=out.mins,
+               clip_counts=clip_counts, dev_status=dev_status)
+    d = out.desc()
+    st = load().sss_quantize_rotated(_ptr(w), block, ctypes.byref(d), _ptr(clip_counts),
+                                     _ptr(dev_status), _stream(stream))
+    _check(fn, st)
+    return out
