@@ -126,6 +126,17 @@ def lib():
             L.orc_quantize_act_q8.restype = i32
             L.orc_gemv_q8.argtypes = [vp, vp, vp, i64, i64, i32, i32, i32, vp, vp, i64, vp]
             L.orc_gemv_q8.restype = None
+            L.orc_fwht_f32.argtypes = [vp, i32]
+            L.orc_fwht_f32.restype = None
+            L.orc_rotate_rows.argtypes = [vp, i64, i64, i32, vp]
+            L.orc_rotate_rows.restype = None
+            L.orc_rotate_cols.argtypes = [vp, i64, i64, i32, vp]
+            L.orc_rotate_cols.restype = None
+            L.orc_lsq_scale.argtypes = [vp, i32, i32, i32, i32, ctypes.c_float]
+            L.orc_lsq_scale.restype = ctypes.c_float
+            L.orc_lsq_quantize.argtypes = [vp, i64, i64, i32, i32, i32, i32, ctypes.c_float,
+                                           vp, vp]
+            L.orc_lsq_quantize.restype = i32
         return _lib
 
 
@@ -288,3 +299,45 @@ def gemv_q8(codes, scales, mins, n: int, k: int, q: int, g: int, grid: int,
     lib().orc_gemv_q8(_p(codes), _p(scales), _p(mins), n, k, q, g, grid, _p(xq), _p(xd),
                       nb, _p(y))
     return y
+
+
+def fwht(x) -> np.ndarray:
+    """Normalized Walsh-Hadamard transform of one fp32 vector (length a
+    power of two): the fp32 fast transform, strides 1, 2, ..., b/2, then
+    times fl32(1/sqrt(b))."""
+    v = np.array(x, np.float32, copy=True)
+    lib().orc_fwht_f32(_p(v), v.size)
+    return v
+
+
+def rotate(W, b: int, side: str = "rows") -> np.ndarray:
+    """W [n, k] fp32 rotated by the normalized Hadamard of block size b on
+    its input side (side="rows": every b-block of a row) or its output side
+    (side="cols": every b-block of a column)."""
+    W = np.ascontiguousarray(W, np.float32)
+    n, k = W.shape
+    out = np.empty_like(W)
+    if side == "rows":
+        assert k % b == 0
+        lib().orc_rotate_rows(_p(W), n, k, b, _p(out))
+    else:
+        assert n % b == 0
+        lib().orc_rotate_cols(_p(W), n, k, b, _p(out))
+    return out
+
+
+def lsq_scale(w, q: int, signed: bool, steps: int, lr: float) -> float:
+    """The LSQ-refined fp32 scale of one group (see orc_lsq_scale)."""
+    w = np.ascontiguousarray(w, np.float32)
+    return float(np.float32(lib().orc_lsq_scale(_p(w), w.size, q, int(signed), steps, lr)))
+
+
+def lsq_quantize(W, q: int, g: int, grid: int, steps: int, lr: float):
+    """Symmetric-grid quantization with LSQ-refined scales: (codes, scales, flags)."""
+    W = np.ascontiguousarray(W, np.float32)
+    n, k = W.shape
+    codes = np.zeros((n, k * q // 8), np.uint8)
+    scales = np.zeros((n, k // g), np.uint16)
+    flags = lib().orc_lsq_quantize(_p(W), n, k, q, g, grid, steps, np.float32(lr), _p(codes),
+                                   _p(scales))
+    return codes, scales, int(flags)

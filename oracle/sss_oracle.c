@@ -411,3 +411,112 @@ void orc_gemv_q8(const uint8_t* codes, const uint16_t* scales,
   }
   free(row);
 }
+
+/* ------------------------------------------------------------------------ */
+/* Normalized Hadamard rotation (Sec. 5 composition; Appendix C).            */
+/* ------------------------------------------------------------------------ */
+
+void orc_fwht_f32(float* x, int32_t b) {
+  for (int32_t h = 1; h < b; h *= 2) {
+    for (int32_t i = 0; i < b; i += 2 * h) {
+      for (int32_t j = i; j < i + h; ++j) {
+        const float a = x[j], c = x[j + h];
+        x[j] = a + c;
+        x[j + h] = a - c;
+      }
+    }
+  }
+  const float norm = (float)(1.0 / sqrt((double)b)); /* the fp32 nearest 1/sqrt(b) */
+  for (int32_t j = 0; j < b; ++j) x[j] = x[j] * norm;
+}
+
+void orc_rotate_rows(const float* W, int64_t n, int64_t k, int32_t b, float* out) {
+  if (out != W) memcpy(out, W, (size_t)n * (size_t)k * sizeof(float));
+  for (int64_t r = 0; r < n; ++r)
+    for (int64_t c0 = 0; c0 < k; c0 += b) orc_fwht_f32(out + r * k + c0, b);
+}
+
+void orc_rotate_cols(const float* W, int64_t n, int64_t k, int32_t b, float* out) {
+  float* col = (float*)malloc((size_t)b * sizeof(float));
+  for (int64_t r0 = 0; r0 < n; r0 += b) {
+    for (int64_t c = 0; c < k; ++c) {
+      for (int32_t i = 0; i < b; ++i) col[i] = W[(r0 + i) * k + c];
+      orc_fwht_f32(col, b);
+      for (int32_t i = 0; i < b; ++i) out[(r0 + i) * k + c] = col[i];
+    }
+  }
+  free(col);
+}
+
+/* ------------------------------------------------------------------------ */
+/* Signed LSQ scale refinement (Sec. 5 learned grids; Appendix C).           */
+/* ------------------------------------------------------------------------ */
+
+float orc_lsq_scale(const float* w, int32_t g, int32_t q, int32_t signed_grid,
+                    int32_t steps, float lr) {
+  orc_group_t info;
+  const int32_t grid = signed_grid ? ORC_GRID_SIGNED_SYM : ORC_GRID_UNSIGNED_SYM;
+  (void)orc_quantize_group(w, g, q, grid, NULL, NULL, NULL, &info);
+  float s = info.s32; /* the (signed) absmax initialisation */
+  if (s == 0.0f) return s;
+  const float qn = (float)(-(1 << (q - 1))), qp = (float)((1 << (q - 1)) - 1);
+  const float gscale = (float)(1.0 / sqrt((double)g * (double)qp)); /* LSQ gradient scale */
+  const float step = lr * gscale;
+  float* t = (float*)malloc((size_t)g * sizeof(float));
+  for (int32_t it = 0; it < steps; ++it) {
+    for (int32_t i = 0; i < g; ++i) {
+      const float v = w[i] / s;
+      float c = rintf(v);
+      float d;
+      if (v <= qn) {
+        c = qn;
+        d = qn;
+      } else if (v >= qp) {
+        c = qp;
+        d = qp;
+      } else {
+        if (c < qn) c = qn; /* v > qn but rint(v) may still equal qn */
+        if (c > qp) c = qp;
+        d = c - v;
+      }
+      const float e = s * c - w[i];
+      t[i] = (2.0f * e) * d;
+    }
+    for (int32_t h = g / 2; h >= 1; h /= 2)
+      for (int32_t i = 0; i < h; ++i) t[i] = t[i] + t[i + h];
+    float sn = s - step * t[0];
+    if (sn * s <= 0.0f) sn = s * 0.5f; /* keep the sign; never reach zero */
+    s = sn;
+  }
+  free(t);
+  return s;
+}
+
+int32_t orc_lsq_quantize(const float* W, int64_t n, int64_t k, int32_t q,
+                         int32_t g, int32_t grid, int32_t steps, float lr,
+                         uint8_t* codes, uint16_t* scales) {
+  int32_t flags = 0;
+  const int64_t ngroups = n * (k / g);
+  const int32_t half = 1 << (q - 1);
+  uint8_t* u = (uint8_t*)malloc((size_t)g);
+  for (int64_t G = 0; G < ngroups; ++G) {
+    const float* w = W + G * g;
+    orc_group_t info;
+    /* NaN/Inf and all-zero groups: the placeholder codes; RANGE is judged
+     * on the refined scale that is stored, below */
+    flags |= orc_quantize_group(w, g, q, grid, NULL, NULL, u, &info) & ORC_FLAG_NONFINITE;
+    const float s = orc_lsq_scale(w, g, q, grid == ORC_GRID_SIGNED_SYM, steps, lr);
+    if (s != 0.0f) {
+      for (int32_t j = 0; j < g; ++j) {
+        int32_t c = (int32_t)orc_rne_quotient(w[j], s);
+        c = clampi(c, -half, half - 1);
+        u[j] = (uint8_t)(c + half);
+      }
+    }
+    scales[G] = orc_f32_to_f16(s);
+    if ((scales[G] & 0x7fffu) == 0x7c00u) flags |= ORC_FLAG_RANGE;
+    orc_pack_group(u, g, q, codes + G * (int64_t)(g * q / 8));
+  }
+  free(u);
+  return flags;
+}

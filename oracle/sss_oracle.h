@@ -136,6 +136,61 @@ void orc_gemv_q8(const uint8_t* codes, const uint16_t* scales,
                  int32_t g, int32_t grid, const int8_t* xq,
                  const uint16_t* xd16, int64_t nb, double* y);
 
+/* ---------------------------------------------------------------------- */
+/* Normalized Hadamard rotation of the weights before quantization (Sec. 5  */
+/* "Composition with PTQ methods"; Appendix C: rotations merged into the    */
+/* weights, grids computed on the rotated weights).                         */
+/* ---------------------------------------------------------------------- */
+
+/* The normalized Walsh-Hadamard transform of x[0..b) (b a power of two,
+ * Sylvester order H_2m = [[H_m, H_m], [H_m, -H_m]]), in the arithmetic this
+ * build takes for it (reading: the paper names the rotation, not its
+ * arithmetic): the in-place fast transform in IEEE fp32 with strides
+ * h = 1, 2, ..., b/2, each butterfly (a, c) -> (a + c, a - c), then every
+ * element times the fp32 nearest to 1/sqrt(b). */
+void orc_fwht_f32(float* x, int32_t b);
+
+/* W [n][k] rotated on its input side, W <- W (I (x) H_b/sqrt(b)): every
+ * block of b consecutive elements of a row transformed as above
+ * (b | k).  out may equal W. */
+void orc_rotate_rows(const float* W, int64_t n, int64_t k, int32_t b, float* out);
+
+/* W [n][k] rotated on its output side, W <- (I (x) H_b/sqrt(b)) W: every
+ * block of b consecutive rows transformed column by column (b | n). */
+void orc_rotate_cols(const float* W, int64_t n, int64_t k, int32_t b, float* out);
+
+/* ---------------------------------------------------------------------- */
+/* Signed LSQ scale refinement (Sec. 5 "Composition with learned rotations  */
+/* and grid parameters"; Appendix C: LSQ with s != 0 for the signed         */
+/* formats, s > 0 for the conventional ones).  The paper learns the scales  */
+/* on calibration data through the model loss; this is the data-free        */
+/* reading on each group's own reconstruction loss (see orc_lsq_scale).     */
+/* ---------------------------------------------------------------------- */
+
+/* The refined scale of one group w[0..g-1] (g a power of two, 32..128):
+ * s_0 = the signed absmax scale gamma* alpha (signed_grid != 0) or the
+ * absmax scale alpha; then `steps` LSQ steps on L(s) = sum (s c_i - w_i)^2,
+ * all in IEEE fp32 without fused multiply-add:
+ *   v_i = w_i / s, c_i = clip(rint(v_i), -2^(q-1), 2^(q-1) - 1),
+ *   d_i = dw^_i/ds, LSQ's straight-through estimate: c_i - v_i when v_i
+ *         lies strictly inside (-2^(q-1), 2^(q-1) - 1), else the clip value,
+ *   e_i = s c_i - w_i,   t_i = (2 e_i) d_i,
+ *   G = sum t_i in the pairwise order: t_i <- t_i + t_{i+h} for
+ *       h = g/2, g/4, ..., 1, G = t_0,
+ *   s' = s - (lr * (1/sqrt(g (2^(q-1) - 1)))) * G  (LSQ's gradient scale),
+ *   and s' keeps the sign of s: if s' s <= 0 then s' = s / 2.
+ * An all-zero (or underflowed) or non-finite group keeps s = 0.  */
+float orc_lsq_scale(const float* w, int32_t g, int32_t q, int32_t signed_grid,
+                    int32_t steps, float lr);
+
+/* Quantize W [n][k] on the symmetric grid with every group's scale refined
+ * by orc_lsq_scale: codes c = clip(RNE(w/s)) of the exact quotient with the
+ * refined fp32 scale s, packed as orc_quantize packs them, fp16 scales.
+ * grid: ORC_GRID_SIGNED_SYM or ORC_GRID_UNSIGNED_SYM.  Returns OR-ed flags. */
+int32_t orc_lsq_quantize(const float* W, int64_t n, int64_t k, int32_t q,
+                         int32_t g, int32_t grid, int32_t steps, float lr,
+                         uint8_t* codes, uint16_t* scales);
+
 #ifdef __cplusplus
 }
 #endif
