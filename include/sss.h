@@ -260,7 +260,8 @@ sss_status_t sss_quantize_act_q8(const uint16_t* x_bf16, int64_t rows, int64_t k
  * every value times the fp32 nearest to 1/sqrt(b).  H_b/sqrt(b) is
  * symmetric and orthogonal: W x = (W R)(R x) for R = I (x) H_b/sqrt(b).
  */
-#define SSS_ROTATE_INPUT 0  /* W <- W R: every block of b consecutive values of a row (b | k) */
+#define SSS_ROTATE_INPUT 0  /* W <- W R: every block of b consecutive values of a row (b | k,
+                               k a multiple of 4)                                            */
 #define SSS_ROTATE_OUTPUT 1 /* W <- R W: every block of b consecutive rows, per column
                                (b | n, and k a multiple of 8192/b)                          */
 
@@ -281,6 +282,30 @@ sss_status_t sss_hadamard(const float* w, float* out, int64_t n, int64_t k,
 sss_status_t sss_quantize_rotated(const float* w, int32_t block, const sss_qtensor_t* out,
                                   uint8_t* clip_counts, uint32_t* dev_status,
                                   void* stream);
+
+/*
+ * sss_quantize_lsq -- symmetric-grid quantization with every group's scale
+ * refined by LSQ steps (Sec. 5 "Composition with learned rotations and grid
+ * parameters"; Appendix C: LSQ, the scale constrained to s != 0 for the
+ * signed formats and s > 0 for the conventional ones).  The paper learns
+ * the scales through the model loss on calibration data; this is the
+ * data-free reading on each group's reconstruction loss L(s) =
+ * sum (s c_i - w_i)^2, in IEEE fp32 without fused multiply-add:
+ *   s_0 = gamma* alpha (SIGNED) or alpha (UNSIGNED), as sss_quantize;
+ *   each step: v_i = w_i / s, c_i = clip(rint(v_i)), d_i = c_i - v_i inside
+ *   the alphabet and the clip value outside (LSQ's straight-through
+ *   derivative of w^_i = s c_i), t_i = (2 (s c_i - w_i)) d_i, G = the
+ *   pairwise sum t_i <- t_i + t_{i+h} (h = g/2, ..., 1),
+ *   s <- s - (lr / sqrt(g (2^(q-1) - 1))) G, and a step that would cross or
+ *   reach zero halves s instead, so the sign is kept;
+ *   then codes c = clip(RNE(w / s)) of the exact quotient and fp16 s, in the
+ *   layout of sss_quantize.  steps = 0 reproduces sss_quantize.
+ *   out   [in]  as sss_quantize; grid SIGNED_SYM or UNSIGNED_SYM.
+ *   steps [in]  >= 0;  lr [in] >= 0.
+ * Errors: SSS_E_ARG, SSS_E_ALIGN, SSS_E_UNSUPPORTED (ASYM), SSS_E_CUDA.
+ */
+sss_status_t sss_quantize_lsq(const float* w, const sss_qtensor_t* out, int32_t steps,
+                              float lr, uint32_t* dev_status, void* stream);
 
 /*
  * sss_sign_diagnostics -- the cardinality margin and the realised l2 gain of

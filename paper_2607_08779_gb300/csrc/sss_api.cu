@@ -296,7 +296,7 @@ sss_status_t sss_hadamard(const float* w, float* out, int64_t n, int64_t k, int3
                           int32_t side, void* stream) {
   if (n < 0 || k < 0 || n > kMaxDim || k > kMaxDim || !pow2_block(block)) return SSS_E_ARG;
   if (side != SSS_ROTATE_INPUT && side != SSS_ROTATE_OUTPUT) return SSS_E_ARG;
-  if (side == SSS_ROTATE_INPUT && k % block != 0) return SSS_E_ARG;
+  if (side == SSS_ROTATE_INPUT && (k % block != 0 || k % 4 != 0)) return SSS_E_ARG;
   if (side == SSS_ROTATE_OUTPUT && (n % block != 0 || k % (8192 / block) != 0)) return SSS_E_ARG;
   if (n == 0 || k == 0) return SSS_OK;
   if (w == nullptr || out == nullptr) return SSS_E_ARG;
@@ -318,6 +318,21 @@ sss_status_t sss_quantize_rotated(const float* w, int32_t block, const sss_qtens
   return finish("sss_quantize_rotated",
                 launch_quantize_rotated(w, block, *out, clip_counts, dev_status,
                                         static_cast<cudaStream_t>(stream)));
+}
+
+sss_status_t sss_quantize_lsq(const float* w, const sss_qtensor_t* out, int32_t steps,
+                              float lr, uint32_t* dev_status, void* stream) {
+  sss_status_t st = check_tensor(out);
+  if (st != SSS_OK) return st;
+  if (out->grid == SSS_GRID_ASYM) return SSS_E_UNSUPPORTED;
+  if (steps < 0 || !(lr >= 0.f) || !(lr < 1e30f)) return SSS_E_ARG;
+  if (out->n == 0 || out->k == 0) return SSS_OK;
+  if (w == nullptr) return SSS_E_ARG;
+  if (!aligned(w, 4) || !aligned(out->codes, 4) || !aligned(out->scales, 2) ||
+      (dev_status && !aligned(dev_status, 4)))
+    return SSS_E_ALIGN;
+  return finish("sss_quantize_lsq", launch_quantize_lsq(w, *out, steps, lr, dev_status,
+                                                        static_cast<cudaStream_t>(stream)));
 }
 
 sss_status_t sss_sign_diagnostics(const float* w, int64_t n, int64_t k, int32_t q,

@@ -58,6 +58,9 @@ cudaError_t launch_hadamard(const float* w, float* out, int64_t n, int64_t k, in
 cudaError_t launch_quantize_rotated(const float* w, int b, const sss_qtensor_t& t, uint8_t* clip,
                                     uint32_t* status, cudaStream_t stream);
 
+cudaError_t launch_quantize_lsq(const float* w, const sss_qtensor_t& t, int steps, float lr,
+                                uint32_t* status, cudaStream_t stream);
+
 cudaError_t launch_sign_diagnostics(const float* w, int64_t n, int64_t k, int q, int g,
                                     int16_t* margin, double* gain, unsigned long long* hist,
                                     uint32_t* status, cudaStream_t stream);

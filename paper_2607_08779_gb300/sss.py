@@ -34,7 +34,7 @@ EXPORTS = ("sss_codes_bytes", "sss_status_string", "sss_last_error", "sss_quanti
            "sss_dequantize", "sss_gemv", "sss_gemv_multi", "sss_gemm", "sss_workspace_bytes",
            "sss_gemm_noalloc", "sss_gemm_noalloc_max_scratch_bytes", "sss_test_set_stall",
            "sss_gemm_q8", "sss_quantize_act_q8", "sss_sign_diagnostics", "sss_hadamard",
-           "sss_quantize_rotated")
+           "sss_quantize_rotated", "sss_quantize_lsq")
 
 GEMV_PDL = 0x1
 GEMV_WEIGHTS_READY = 0x2
@@ -123,6 +123,8 @@ def load(build_if_needed: bool = True):
         L.sss_hadamard.restype = i32
         L.sss_quantize_rotated.argtypes = [vp, i32, P, vp, vp, vp]
         L.sss_quantize_rotated.restype = i32
+        L.sss_quantize_lsq.argtypes = [vp, P, i32, ctypes.c_float, vp, vp]
+        L.sss_quantize_lsq.restype = i32
         L.sss_test_set_stall.argtypes = [ctypes.c_uint32]
         L.sss_test_set_stall.restype = None
         _lib = L
@@ -476,5 +478,25 @@ def sss_quantize_rotated(w, block: int, q: int, group: int, grid: int,
     d = out.desc()
     st = load().sss_quantize_rotated(_ptr(w), block, ctypes.byref(d), _ptr(clip_counts),
                                      _ptr(dev_status), _stream(stream))
+    _check(fn, st)
+    return out
+
+
+def sss_quantize_lsq(w, q: int, group: int, grid: int, steps: int, lr: float,
+                     out: Optional["QTensor"] = None, dev_status=None, stream=None) -> "QTensor":
+    """Symmetric-grid quantization of fp32 w [n, k] with LSQ-refined scales."""
+    import torch
+
+    n, k = w.shape
+    fn = "sss_quantize_lsq"
+    _need(fn, "w", w, torch.float32, n * k)
+    if out is None:
+        out = empty_qtensor(n, k, q, group, grid, device=w.device)
+    _need_qtensor(fn, out)
+    _need_status(fn, dev_status)
+    _on_device(fn, w=w, codes=out.codes, scales=out.scales, dev_status=dev_status)
+    d = out.desc()
+    st = load().sss_quantize_lsq(_ptr(w), ctypes.byref(d), int(steps), float(lr),
+                                 _ptr(dev_status), _stream(stream))
     _check(fn, st)
     return out
