@@ -156,9 +156,11 @@ __device__ __forceinline__ void store_run(uint8_t* __restrict__ codes, int64_t g
 // run index gr in the flat weight array) together with the other runs of
 // its group (the L = G/32 consecutive lanes of the warp): group max / min,
 // scale, codes, packing, scale / min / clip-count stores.  Every lane of
-// the warp calls it (valid = false for lanes past the last run).
-template <int Q, int GRID, int G, bool STATS>
-__device__ __forceinline__ void quantize_run(float (&x)[32], int r, bool valid, int64_t gr,
+// the warp calls it (valid = false for lanes past the last run).  wat(e)
+// re-reads x[e] as it was passed in (the rare exact-tie decisions use it,
+// so x need not stay live in registers).
+template <int Q, int GRID, int G, bool STATS, class Wat>
+__device__ __forceinline__ void quantize_run(float (&x)[32], Wat wat, int r, bool valid, int64_t gr,
                                              uint8_t* __restrict__ codes,
                                              uint16_t* __restrict__ scales,
                                              uint16_t* __restrict__ mins,
@@ -170,18 +172,15 @@ __device__ __forceinline__ void quantize_run(float (&x)[32], int r, bool valid, 
   constexpr int OFF = (GRID == SSS_GRID_ASYM) ? 0 : HALF;
   const int64_t grp = gr / L;
   const int lg = static_cast<int>(gr % L);
-  float mx = x[0], mn = x[0], sum = 0.f;
+  // max with NaN propagation: a NaN anywhere makes mx NaN, an infinity
+  // makes mx or mn infinite, so the run is non-finite iff they are
+  float mx = x[0], mn = x[0];
 #pragma unroll
   for (int e = 0; e < 32; ++e) {
-    mx = fmaxf(mx, x[e]);
+    asm("max.NaN.f32 %0, %0, %1;" : "+f"(mx) : "f"(x[e]));
     mn = fminf(mn, x[e]);
-    sum += x[e];  // NaN/Inf anywhere -> non-finite sum (checked exactly below)
   }
-  unsigned bad = 0;
-  if (is_nonfinite(sum)) {
-#pragma unroll
-    for (int e = 0; e < 32; ++e) bad |= is_nonfinite(x[e]);
-  }
+  unsigned bad = (is_nonfinite(mx) || is_nonfinite(mn)) ? 1u : 0u;
 #pragma unroll
   for (int o = L / 2; o >= 1; o >>= 1) {
     mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
@@ -206,26 +205,31 @@ __device__ __forceinline__ void quantize_run(float (&x)[32], int r, bool valid, 
 #pragma unroll
       for (int e = 0; e < 32; ++e) u[e] = HALF;
     } else {
-      float ss = s;
+      float ss = s, sig = 1.f;
       // alpha is an exact power-of-two scaling of M unless it is
-      // subnormal; then |w/s| may exceed 2^(q-1) slightly and both ends clip
-      int lo_clip = 0x80000000;
-      if (M < 0x1p-96f || M > 0x1p+96f) {  // keep 1/s normal: scale w and s by 2^+-64
-        const float sig = (M < 1.f) ? 0x1p+64f : 0x1p-64f;
+      // subnormal; then |w/s| may exceed 2^(q-1) slightly and both ends
+      // clip (otherwise c_pre >= -2^(q-1) and only +2^(q-1) leaves A_q)
+      const bool lo_clip = M < 0x1p-96f || M > 0x1p+96f;
+      if (lo_clip) {  // keep 1/s normal: scale w and s by 2^+-64
+        sig = (M < 1.f) ? 0x1p+64f : 0x1p-64f;
         ss = __fmul_rn(s, sig);
 #pragma unroll
         for (int e = 0; e < 32; ++e) x[e] = __fmul_rn(x[e], sig);
-        lo_clip = 0;
       }
       const float rc = __frcp_rn(ss);
+      // c_pre + 2^(q-1); w * 1 is w, so the re-read matches x in both cases
+      codes_of<OFF>(x, ss, rc, u, [&](int e) { return __fmul_rn(wat(e), sig); });
 #pragma unroll
       for (int e = 0; e < 32; ++e) {
-        const int up = code_of<OFF>(x[e], ss, rc);  // c_pre + 2^(q-1)
         if constexpr (STATS) {
-          n_self += (up == 2 * HALF);  // c_pre == +2^(q-1): in C_gamma
-          n_other += (up == 0);        // c_pre == -2^(q-1): in C_-gamma
+          n_self += (u[e] == 2 * HALF);  // c_pre == +2^(q-1): in C_gamma
+          n_other += (u[e] == 0);        // c_pre == -2^(q-1): in C_-gamma
         }
-        u[e] = max(min(up, UMAX), lo_clip);  // normally only +2^(q-1) leaves A_q
+        u[e] = min(u[e], UMAX);
+      }
+      if (lo_clip) {
+#pragma unroll
+        for (int e = 0; e < 32; ++e) u[e] = max(u[e], 0);
       }
     }
     s16 = __half_as_ushort(__float2half_rn(s));
@@ -255,10 +259,15 @@ __device__ __forceinline__ void quantize_run(float (&x)[32], int r, bool valid, 
       const float rc = __frcp_rn(ss);
 #pragma unroll
       for (int e = 0; e < 32; ++e) {
-        float d = __fsub_rn(x[e], mn);  // fl32(w - min) >= 0
-        if (sig != 1.f) d = __fmul_rn(d, sig);
-        u[e] = min(code_of<0>(d, ss, rc), UMAX);
+        x[e] = __fsub_rn(x[e], mn);  // fl32(w - min) >= 0
+        if (sig != 1.f) x[e] = __fmul_rn(x[e], sig);
       }
+      codes_of<0>(x, ss, rc, u, [&](int e) {
+        const float d = __fsub_rn(wat(e), mn);
+        return sig != 1.f ? __fmul_rn(d, sig) : d;
+      });
+#pragma unroll
+      for (int e = 0; e < 32; ++e) u[e] = min(u[e], UMAX);
     }
     s16 = __half_as_ushort(__float2half_rn(s));  // inf when the step overflowed
     m16 = __half_as_ushort(__float2half_rn(mn));
@@ -361,12 +370,24 @@ __global__ void __launch_bounds__(kQThreads, 1)
                        : "r"(run_a + 16u * static_cast<uint32_t>((j + r) & 7)));
         x[4 * j] = v.x; x[4 * j + 1] = v.y; x[4 * j + 2] = v.z; x[4 * j + 3] = v.w;
       }
+      // the stage is released after the run is quantized: the rare exact
+      // tie decisions re-read their weights from it
+      quantize_run<Q, GRID, G, STATS>(
+          x,
+          [&](int e) {
+            float v = 0.f;
+            if (valid)
+              asm volatile("ld.shared.f32 %0, [%1];"
+                           : "=f"(v)
+                           : "r"(run_a + 16u * static_cast<uint32_t>(((e >> 2) + r) & 7) +
+                                 4u * static_cast<uint32_t>(e & 3)));
+            return v;
+          },
+          r, valid, w0 / 32 + sl, codes, scales, mins, clip, status);
       __syncwarp();
       if (lane == 0)
         asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(q_su32(&empty[s]))
                      : "memory");
-      quantize_run<Q, GRID, G, STATS>(x, r, valid, w0 / 32 + sl, codes, scales, mins, clip,
-                                      status);
     }
   }
   __syncthreads();
@@ -501,8 +522,14 @@ __global__ void __launch_bounds__(kRotThreads)
       x[4 * j] = __fmul_rn(v.x, norm); x[4 * j + 1] = __fmul_rn(v.y, norm);
       x[4 * j + 2] = __fmul_rn(v.z, norm); x[4 * j + 3] = __fmul_rn(v.w, norm);
     }
+    quantize_run<Q, GRID, G, STATS>(
+        x,
+        [&](int e) {
+          return __fmul_rn(reinterpret_cast<const float*>(run)[4 * (((e >> 2) + r) & 7) + (e & 3)],
+                           norm);
+        },
+        r, valid, w0 / 32 + sl, codes, scales, mins, clip, status);
     __syncthreads();  // the chunk is read: the next one may overwrite it
-    quantize_run<Q, GRID, G, STATS>(x, r, valid, w0 / 32 + sl, codes, scales, mins, clip, status);
   }
 }
 
