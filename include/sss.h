@@ -72,8 +72,8 @@ typedef enum {
                                    for symmetric grids, u = 0 and s = +0 for ASYM)     */
 #define SSS_FLAG_RANGE 0x2u     /* a stored fp16 scale or min is infinite (|s| >= 65520),
                                    or the fp32 ASYM step overflowed (codes then 0)     */
-#define SSS_FLAG_TIMEOUT 0x4u   /* a bounded pipeline wait (sss_gemm, or the batch-1
-                                   streaming GEMV) expired; the output is incomplete  */
+#define SSS_FLAG_TIMEOUT 0x4u   /* a bounded pipeline wait (sss_gemm, or the batched
+                                   GEMV) expired; the output is incomplete            */
 
 typedef enum { SSS_OUT_F32 = 0, SSS_OUT_F16 = 1, SSS_OUT_BF16 = 2 } sss_dtype_t;
 
@@ -188,7 +188,8 @@ sss_status_t sss_gemv(const sss_qtensor_t* qt, const uint16_t* x_bf16,
  *   count   [in]  1..4.
  *   x_bf16  [in]  device bf16 [k], 16-byte aligned.
  *   flags   [in]  SSS_GEMV_* bits.
- *   dev_status [out] nullable; SSS_FLAG_TIMEOUT if a bounded wait expired.
+ *   dev_status [out] nullable; with SSS_GEMV_ACT_Q8 the Q8_0 flags of x
+ *                 (the streaming kernel has no waits that could time out).
  * Shapes with k % 256 != 0 or k % (8*group) != 0, or unaligned buffers, run
  * as one sss_gemv per matrix (flags then have no effect, and SSS_GEMV_ACT_Q8
  * returns SSS_E_UNSUPPORTED).
@@ -361,17 +362,18 @@ size_t sss_gemm_noalloc_max_scratch_bytes(void);
 /*
  * sss_test_set_stall -- test hook for the bounded waits; the paper has no
  * counterpart.  While a bit below is set, every later launch of that kernel
- * family leaves one mbarrier one arrive short: the batch-1 GEMV and the
- * batched GEMV on the first output tile's partial sums (only where a tile's
- * k-range is split across several warps), the GEMM on the first stage's
- * weight tile.  The wait on that barrier then runs out after its bound
+ * family leaves one mbarrier one arrive short: the batched GEMV on the first
+ * output tile's partial sums (only where a tile's k-range is split across
+ * several warps), the GEMM on the first stage's weight tile.  The batch-1
+ * streaming GEMV has no data-dependent waits (its warps meet only at
+ * CTA-wide barriers), so its bit has no effect.  The wait on that barrier then runs out after its bound
  * (about one second), the kernel raises SSS_FLAG_TIMEOUT in dev_status,
  * lets its own copies and MMAs in flight finish, releases its tensor memory
  * and returns; its output is incomplete.  Nothing faults or hangs.
  * mask = 0 (the default) restores normal launches.  Process-wide; affects
  * launches issued (or captured) after the call on every thread.
  */
-#define SSS_TEST_STALL_GEMV 0x1u       /* gemv_stream_kernel (sss_gemv batch 1, sss_gemv_multi) */
+#define SSS_TEST_STALL_GEMV 0x1u       /* gemv_stream_kernel: no waits, no effect               */
 #define SSS_TEST_STALL_GEMV_BATCH 0x2u /* gemv_batch_kernel (sss_gemv batch 2..16)             */
 #define SSS_TEST_STALL_GEMM 0x4u       /* gemm_kernel (sss_gemm, sss_gemm_noalloc)             */
 void sss_test_set_stall(uint32_t mask);

@@ -23,15 +23,16 @@
 //    registers; a slot is refilled as soon as its unit is multiplied, and
 //    the whole ring is filled before the grid-dependency wait.  Shared
 //    memory holds only the activation operand.
-//  * with KW > 1 a tile's partials meet in a double-buffered shared array
-//    behind mbarriers and only the reducing warp waits; with KW = 1 a warp
-//    owns whole tiles and writes y directly.
+//  * with KW > 1 every warp leaves its row partials of each of its tiles in
+//    its own slot of a shared array, with no wait; after the last unit the
+//    CTA sums each tile's KW partials in warp order and stores y.  With
+//    KW = 1 a warp owns whole tiles and writes y directly.
 //
 // The activation vector is staged once per CTA, after the grid-dependency
 // wait of a programmatic dependent launch (weights may be prefetched before
-// it only when the caller states they are not written upstream).  Every
-// mbarrier wait is bounded; on expiry the kernel raises SSS_FLAG_TIMEOUT and
-// winds down without further waits.
+// it only when the caller states they are not written upstream).  The
+// kernel has no data-dependent waits: its only synchronisation is two
+// CTA-wide barriers (after staging x, and before the final sums).
 #include <cuda.h>
 
 #include <stdint.h>
@@ -239,7 +240,7 @@ struct StreamArgs {
   int lgkw;            // log2(warps per tile)
   int early_weights;   // prefetch weights before the grid-dependency wait
   int act_q8;          // quantize the activations to Q8_0 while staging them
-  int stall;           // test hook: one partial of the first tile is never announced
+  int rounds;          // tiles per warp group at most (the partial array's depth)
   uint32_t* status;
 };
 
@@ -259,14 +260,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   // ---- shared memory carve-up ----
   // staged activations [nsc][64 B] | two 64-byte zero blocks, the first 128
   // bytes past a 128-aligned offset (the B operand of lanes that carry no
-  // data; see compute) | per-sub-chunk {b, f} | barriers | partials | flag
+  // data; see compute) | per-sub-chunk {b, f} | row partials (KW > 1)
   unsigned char* xs = smem;
   const uint32_t zoff = (static_cast<uint32_t>(nsc) * 64u + 127u) & ~127u;
   float2* sbf = reinterpret_cast<float2*>(xs + zoff + 128);              // [nsc]
-  uint64_t* pready = reinterpret_cast<uint64_t*>(sbf + nsc);              // [kWarps][2]
-  uint64_t* pfree = pready + 2 * kWarps;                                   // [kWarps][2]
-  float* part = reinterpret_cast<float*>(pfree + 2 * kWarps);              // [kWarps][2][R]
-  volatile int* abort = reinterpret_cast<volatile int*>(part + 2 * kWarps * R);
+  float* part = reinterpret_cast<float*>(sbf + nsc);                      // [ngrp][rounds][KW][R]
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -274,14 +272,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   const int grp = warp >> lgkw;        // this warp's group (one tile at a time)
   const int kw = warp & (KW - 1);      // its share of the tile's k-range
 
-  if (threadIdx.x == 0) {
-    for (int i = 0; i < 2 * kWarps; ++i) {
-      bar_init(&pready[i], KW * 8);  // the 8 quad leaders of every warp of a group
-      bar_init(&pfree[i], 1);
-    }
-    *abort = 0;
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  }
   if (threadIdx.x >= 32 && threadIdx.x < 64)
     reinterpret_cast<uint32_t*>(xs + zoff)[threadIdx.x - 32] = 0u;  // the zero blocks
   // allow the next kernel in the stream to be scheduled as SMs free up
@@ -406,7 +396,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
   stage_x<Q, ASYM>(a.x, nsc, su32(xs), sbf, threadIdx.x, kThreads, a.act_q8 != 0, a.status);
   __syncthreads();
 
-  bool ok = true;
   float acc[2] = {0.f, 0.f};
   // Column gq of B carries sub-chunk 8u + gq of the unit in the mmas of
   // parity h = gq & 1, from the one lane of quad gq >> 1 whose own A rows
@@ -487,12 +476,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
     xl += static_cast<uint32_t>(8 * 64 * KW);
     bl += static_cast<uint32_t>(8 * 8 * KW);
   };
+  // End of the compute cursor's tile i: the warp's two row partials (rows
+  // gq and gq + 8, summed over the quad) go straight to y (KW = 1) or to the
+  // warp's slot of the partial array (KW > 1), summed after the last unit.
   auto tile_end = [&](int64_t i) {
-    const int64_t t = tfirst + i * tstride;
-    int j = 0;
-    while (j + 1 < a.njobs && t >= a.job[j + 1].tile0) ++j;
-    const StreamJob& jb = a.job[j];
-    const int64_t row0 = (t - jb.tile0) * R;
     float v[2];
 #pragma unroll
     for (int hh = 0; hh < 2; ++hh) {
@@ -502,48 +489,25 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
       v[hh] = x;
       acc[hh] = 0.f;
     }
+    if (tq != 0) return;
     if (KW == 1) {
-      if (tq == 0) {
+      const int64_t t = tfirst + i * tstride;
+      int j = 0;
+      while (j + 1 < a.njobs && t >= a.job[j + 1].tile0) ++j;
+      const StreamJob& jb = a.job[j];
+      const int64_t row0 = (t - jb.tile0) * R;
 #pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-          const int64_t r = row0 + gq + 8 * hh;
-          if (r < jb.n) jb.y[r] = v[hh];
-        }
+      for (int hh = 0; hh < 2; ++hh) {
+        const int64_t r = row0 + gq + 8 * hh;
+        if (r < jb.n) jb.y[r] = v[hh];
       }
       return;
     }
-    // the group's KW partials meet behind mbarriers; only the reducing warp
-    // (kw == i % KW) waits for them
-    const int b = static_cast<int>(i & 1);
-    const uint32_t use = static_cast<uint32_t>(i >> 1) & 1u;
-    float* pb = part + (static_cast<size_t>(grp) * 2 + b) * KW * R;
-    uint64_t* rdy = &pready[grp * 2 + b];
-    uint64_t* fre = &pfree[grp * 2 + b];
-    if (tq == 0) {
-      if (!bar_wait(fre, use ^ 1u, abort)) ok = false;
-      pb[kw * R + gq] = v[0];
-      pb[kw * R + gq + 8] = v[1];
-      // (sss_test_set_stall: the last warp's first quad leaves the first
-      // tile's barrier one arrive short, so its reducer's wait runs out)
-      if (!(a.stall && i == 0 && kw == KW - 1 && gq == 0)) bar_arrive(rdy);
-    }
-    if (kw == static_cast<int>(i & (KW - 1))) {
-      if (!bar_wait(rdy, use, abort)) ok = false;
-      if (lane < R) {
-        float sum = 0.f;
-        for (int c = 0; c < KW; ++c) sum += pb[c * R + lane];
-        const int64_t r = row0 + lane;
-        if (r < jb.n && ok) jb.y[r] = sum;
-      }
-      __syncwarp();
-      if (lane == 0) bar_arrive(fre);
-    }
+    float* pb = part + ((static_cast<size_t>(grp) * a.rounds + i) * KW + kw) * R;
+    pb[gq] = v[0];
+    pb[gq + 8] = v[1];
   };
 
-  // warps without units still take part in every tile's reduction
-  if (upw == 0) {
-    for (int64_t i = 0; i < my_tiles; ++i) tile_end(i);
-  }
   // the units, D at a time so the register ring is indexed at compile time;
   // unit k + D - 1 is loaded while unit k is computed
   auto after_unit = [&]() {
@@ -575,20 +539,39 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_stream_kernel(const __grid_c
       }
     }
   }
-  if (*abort && threadIdx.x == 0 && a.status != nullptr) atomicOr(a.status, SSS_FLAG_TIMEOUT);
+  if (KW == 1) return;
+  // ---- the sums of the tiles' KW partials, in warp order (warps without
+  // units left no partial) ----
+  __syncthreads();
+  const int kwn = KW < nunits ? KW : nunits;
+  const int per_grp = a.rounds * R;
+  for (int idx = threadIdx.x; idx < ngrp * per_grp; idx += kThreads) {
+    const int g = idx / per_grp, i = (idx / R) % a.rounds, row = idx % R;
+    const int64_t t = (static_cast<int64_t>(i) * ngrp + g) * gridDim.x + blockIdx.x;
+    if (t >= a.ntiles) continue;
+    int j = 0;
+    while (j + 1 < a.njobs && t >= a.job[j + 1].tile0) ++j;
+    const int64_t r = (t - a.job[j].tile0) * R + row;
+    if (r >= a.job[j].n) continue;
+    const float* pb = part + (static_cast<size_t>(g) * a.rounds + i) * KW * R + row;
+    float sum = 0.f;
+    for (int c = 0; c < kwn; ++c) sum += pb[c * R];
+    a.job[j].y[r] = sum;
+  }
 }
 
-// activations (rounded up to 128) | zero blocks | {b, f} | 4*kWarps
-// barriers | partials | flag
-size_t smem_bytes(int64_t k) {
+// activations (rounded up to 128) | zero blocks | {b, f} | row partials
+// (rounds x 1 KB when KW > 1)
+size_t smem_bytes(int64_t k, int rounds = 0) {
   const int64_t nsc = k / 32;
-  return static_cast<size_t>((nsc * 64 + 127) / 128 * 128 + 128 + 8 * nsc) + 8 * 4 * kWarps +
-         4 * 2 * kWarps * 16 + 16;
+  return static_cast<size_t>((nsc * 64 + 127) / 128 * 128 + 128 + 8 * nsc) +
+         static_cast<size_t>(rounds) * kWarps * 16 * 4;
 }
+constexpr size_t kSmemMax = 227 * 1024;
 
 template <int Q, bool ASYM, int G, int D>
 cudaError_t launch_d(StreamArgs& a, int grid, bool pdl, cudaStream_t stream) {
-  const size_t smem = smem_bytes(a.k);
+  const size_t smem = smem_bytes(a.k, a.lgkw > 0 ? a.rounds : 0);
   auto kern = gemv_stream_kernel<Q, ASYM, G, D>;
   cudaError_t e = ensure_smem(kern, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
@@ -607,7 +590,7 @@ cudaError_t launch_d(StreamArgs& a, int grid, bool pdl, cudaStream_t stream) {
 
 template <int Q, bool ASYM, int G>
 cudaError_t launch_g(StreamArgs& a, int grid, bool pdl, cudaStream_t stream) {
-  if (smem_bytes(a.k) > 227 * 1024) return cudaErrorNotSupported;
+  if (smem_bytes(a.k, a.lgkw > 0 ? a.rounds : 0) > kSmemMax) return cudaErrorNotSupported;
   return launch_d<Q, ASYM, G, 2>(a, grid, pdl, stream);
 }
 
@@ -623,7 +606,8 @@ cudaError_t launch_q(const sss_qtensor_t* const* ts, StreamArgs& a, bool pdl,
   // One CTA per SM (fewer when there are fewer tiles); CTA c takes tiles
   // c, c + grid, ...  Warps per tile: the power of two that minimises the
   // busiest warp's units (rounds of that CTA's tiles x units per warp per
-  // tile), preferring fewer warps per tile (less reduction) on ties.
+  // tile), preferring fewer warps per tile (less reduction) on ties, among
+  // those whose partial array fits in shared memory (KW = 1 needs none).
   const int sms = device_sm_count();
   const int64_t nunits = a.k / 256;
   const int grid = static_cast<int>(std::min<int64_t>(sms, tiles));
@@ -634,13 +618,17 @@ cudaError_t launch_q(const sss_qtensor_t* const* ts, StreamArgs& a, bool pdl,
     const int kwn = 1 << lg;
     if (kwn > 1 && kwn > nunits) break;
     const int64_t ngrp = kWarps >> lg;
-    const int64_t cost = ((per_cta + ngrp - 1) / ngrp) * ((nunits + kwn - 1) / kwn);
+    const int64_t rounds = (per_cta + ngrp - 1) / ngrp;
+    if (lg > 0 && smem_bytes(a.k, static_cast<int>(std::min<int64_t>(rounds, 1 << 20))) > kSmemMax)
+      continue;
+    const int64_t cost = rounds * ((nunits + kwn - 1) / kwn);
     if (cost < best_cost) {
       best_cost = cost;
       best = lg;
     }
   }
   a.lgkw = best;
+  a.rounds = static_cast<int>((per_cta + (kWarps >> best) - 1) / (kWarps >> best));
   switch (ts[0]->group) {
     case 32: return launch_g<Q, ASYM, 32>(a, grid, pdl, stream);
     case 64: return launch_g<Q, ASYM, 64>(a, grid, pdl, stream);
@@ -674,7 +662,6 @@ cudaError_t launch_gemv_stream(const sss_qtensor_t* const* ts, float* const* ys,
   a.k = ts[0]->k;
   a.early_weights = (flags & SSS_GEMV_WEIGHTS_READY) ? 1 : 0;
   a.act_q8 = (flags & SSS_GEMV_ACT_Q8) ? 1 : 0;
-  a.stall = (test_stall_mask() & SSS_TEST_STALL_GEMV) ? 1 : 0;
   a.status = status;
   for (int j = 0; j < count; ++j) {
     a.job[j].codes = ts[j]->codes;
