@@ -70,8 +70,12 @@ typedef enum {
 #define SSS_FLAG_NONFINITE 0x1u /* a weight group contains NaN or +-Inf; that group's
                                    codes/scale are placeholders (u = 2^(q-1) and s = +0
                                    for symmetric grids, u = 0 and s = +0 for ASYM)     */
-#define SSS_FLAG_RANGE 0x2u     /* a stored fp16 scale or min is infinite (|s| >= 65520),
-                                   or the fp32 ASYM step overflowed (codes then 0)     */
+#define SSS_FLAG_RANGE 0x2u     /* sss_quantize: a stored fp16 scale or min is infinite
+                                   (|s| >= 65520), or the fp32 ASYM step overflowed
+                                   (codes then 0).  sss_gemv at batch 2..16 and
+                                   sss_gemm: a group's fp16 weight operand may overflow
+                                   (see those calls); their outputs may then hold
+                                   inf or NaN                                         */
 #define SSS_FLAG_TIMEOUT 0x4u   /* a bounded pipeline wait (sss_gemm, or the batched
                                    GEMV) expired; the output is incomplete            */
 
@@ -144,8 +148,12 @@ sss_status_t sss_dequantize(const sss_qtensor_t* qt, void* out,
  * integer codes meet the activations exactly and the group scale is applied
  * in fp32.  At batch 2..16 (k a multiple of 256), the batch fills the
  * tensor-core columns, so each weight enters the product as w^ rounded once
- * to fp16 (<= 2^-11 relative, as in sss_gemm); that operand overflows if
- * |w^| * 16 >= 65504.
+ * to fp16 (<= 2^-11 relative, as in sss_gemm), times 2^p (p = 0, 2 or 4, the
+ * bit offset of the code's field).  That operand fits fp16 while
+ * |w^| * 2^p < 65520; every group whose scale could break this raises
+ * SSS_FLAG_RANGE (checked per scale, conservatively: |s| * 2^(q-1) * 16 >=
+ * 65520 for the symmetric grids, (|s| * (2^q - 1) + |m|) * 16 >= 65520 for
+ * ASYM).
  *   qt        [in]  packed tensor; codes 16-byte aligned, scales/mins 4-byte
  *                   aligned.
  *   x_bf16    [in]  device bf16 [batch][k], 16-byte aligned.
@@ -154,7 +162,8 @@ sss_status_t sss_dequantize(const sss_qtensor_t* qt, void* out,
  *   workspace [in]  device scratch of ws_bytes >= sss_workspace_bytes(qt,
  *                   batch, SSS_OP_GEMV) bytes, 16-byte aligned, or NULL when
  *                   that size is 0.  Its contents on entry are ignored.
- *   dev_status [out] nullable; SSS_FLAG_TIMEOUT if a bounded wait expired.
+ *   dev_status [out] nullable; SSS_FLAG_TIMEOUT if a bounded wait expired,
+ *                   SSS_FLAG_RANGE as above (batch 2..16).
  * Errors: SSS_E_ARG, SSS_E_ALIGN, SSS_E_WORKSPACE, SSS_E_CUDA.
  */
 sss_status_t sss_gemv(const sss_qtensor_t* qt, const uint16_t* x_bf16,
@@ -204,14 +213,18 @@ sss_status_t sss_gemv_multi(const sss_qtensor_t* const* qts, float* const* ys,
  * prefill is the phase where the matrix products set the time), dequantising
  * weight tiles on chip and accumulating on the tcgen05 tensor cores in fp32
  * (tensor memory).  Tile operands are fp16: w^ rounded to fp16 and X
- * converted from bf16 (exact for 2^-17 <= |x| <= 65504).
+ * converted from bf16 (exact for 2^-17 <= |x| <= 65504).  The weight
+ * operand fits fp16 while |w^| < 65520; every group whose scale could break
+ * this raises SSS_FLAG_RANGE (checked per scale, conservatively: |s| *
+ * 2^(q-1) >= 65520, or |s| * (2^q - 1) + |m| >= 65520 for ASYM).
  *   qt        [in]  packed tensor, symmetric grids or ASYM; k % 64 == 0;
  *                   codes 16-byte aligned.
  *   x_bf16    [in]  device bf16 [m][k], 16-byte aligned.
  *   m         [in]  0 .. 2^24 tokens.
  *   y         [out] device fp32 [m][n], 16-byte aligned, n % 4 == 0.
  *   workspace [in]  as for sss_gemv with SSS_OP_GEMM.
- *   dev_status [out] nullable; SSS_FLAG_TIMEOUT if a bounded wait expired.
+ *   dev_status [out] nullable; SSS_FLAG_TIMEOUT if a bounded wait expired,
+ *                   SSS_FLAG_RANGE as above.
  * Errors: SSS_E_ARG, SSS_E_ALIGN, SSS_E_UNSUPPORTED, SSS_E_WORKSPACE, SSS_E_CUDA.
  */
 sss_status_t sss_gemm(const sss_qtensor_t* qt, const uint16_t* x_bf16,

@@ -22,7 +22,9 @@
 //              each thread owns one weight row of the tile and one 32-code
 //              half of its set's 64-wide k-blocks, loads those codes
 //              and their scale, forms fp16 s*c in natural k order and stores
-//              it with the 128B swizzle the shared-memory descriptor expects;
+//              it with the 128B swizzle the shared-memory descriptor expects
+//              (a group whose scale lets s*c reach 65520, checked per scale
+//              as |s| 2^(q-1) or |s| (2^q - 1) + |m|, raises SSS_FLAG_RANGE);
 //              after the last k-block the same warps drain the fp32
 //              accumulator with tcgen05.ld (each set of four warps one
 //              quarter of the columns) and store Y (for a fixed token, a warp writes
@@ -374,6 +376,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // the global loads run kPrefetch of this thread's k-blocks ahead of use
     constexpr int kPrefetch = 4;
     KBlock ring[kPrefetch];
+    bool big = false;  // a group whose s*c may leave the fp16 range
 #pragma unroll
     for (int q0 = 0; q0 < kPrefetch; ++q0) fetch(ring[q0], set + kDqSets * q0);
     bool ok = true;
@@ -393,9 +396,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           const __half sh = __ushort_as_half(ring[q0].s);
           const __half2 s2 = __halves2half2(sh, sh);
           __half2 m2 = __float2half2_rn(0.f);
+          const float sa = fabsf(__half2float(sh));
+          if constexpr (!ASYM) big |= sa * static_cast<float>(1 << (Q - 1)) >= 65520.f;
           if constexpr (ASYM) {
             const __half mh = __ushort_as_half(ring[q0].m);
             m2 = __halves2half2(mh, mh);
+            big |= sa * static_cast<float>((1 << Q) - 1) + fabsf(__half2float(mh)) >= 65520.f;
           }
           uint32_t u[16];
           code_pairs<Q>(ring[q0].w, u);
@@ -426,6 +432,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         fetch(ring[q0], kb + kDqSets * kPrefetch);
       }
     }
+    if (__any_sync(0xffffffffu, big) && lane == 0 && a.status != nullptr)
+      atomicOr(a.status, SSS_FLAG_RANGE);
     // ---------------- epilogue ----------------
     // a warp may read tensor-memory lanes 32*(warp % 4) .. +31; the four
     // sets of four warps take one quarter of the columns each

@@ -12,7 +12,9 @@
 //    offset 2^(q-1)*2^p, one HMUL2 applies the group scale (min-max grid:
 //    HFMA2 with the scale and the min times 2^p).  The operand is
 //    fp16(w^ * 2^p): the weight rounded once to fp16 (<= 2^-11 relative, as
-//    in sss_gemm), and bounded by |w^| * 16 < 65504;
+//    in sss_gemm).  It fits fp16 while |w^| * 16 < 65520; a group whose
+//    scale lets its codes pass that bound raises SSS_FLAG_RANGE (checked per
+//    scale, conservatively: (|s| 2^(q-1), or |s| (2^q - 1) + |m|) * 16);
 //  * x is staged per K slab in shared memory in mma-B order, pre-divided by
 //    2^p, as fp16, one 8-column block per 8 batch rows (rows past the batch
 //    are zero);
@@ -318,6 +320,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_batch_kernel(const __grid_co
     off[i] = *reinterpret_cast<uint32_t*>(&hv);
   }
 
+  // a group of this thread's whose operand may leave the fp16 range
+  bool big = false;
   auto compute = [&](const Regs& rg, int ul) {
     const uint32_t xu = xs_a + static_cast<uint32_t>(ul * XU);
 #pragma unroll
@@ -328,8 +332,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_batch_kernel(const __grid_co
       for (int hh = 0; hh < 2; ++hh) {
         const uint32_t sb = G == 32 ? ((rg.s[hh] >> (16 * h)) & 0xFFFFu) : (rg.s[hh] & 0xFFFFu);
         S[hh] = f16x2_of(sb);
+        const float sa = fabsf(__half2float(__ushort_as_half(static_cast<unsigned short>(sb))));
+        if constexpr (!ASYM) big |= sa * static_cast<float>(HALF * 16) >= 65520.f;
         if constexpr (ASYM) {
           const uint32_t mb = G == 32 ? ((rg.m[hh] >> (16 * h)) & 0xFFFFu) : (rg.m[hh] & 0xFFFFu);
+          const float ma = fabsf(__half2float(__ushort_as_half(static_cast<unsigned short>(mb))));
+          big |= (sa * static_cast<float>(2 * HALF - 1) + ma) * 16.f >= 65520.f;
 #pragma unroll
           for (int i = 0; i < 3; ++i) M[hh][i] = i == 0 ? f16x2_of(mb) : f16x2_scaled(mb, 2 * i);
         }
@@ -430,6 +438,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_batch_kernel(const __grid_co
       tile_end(s, i);
     }
   }
+  if (__any_sync(0xffffffffu, big) && lane == 0 && a.status != nullptr)
+    atomicOr(a.status, SSS_FLAG_RANGE);
   if (*abort && threadIdx.x == 0 && a.status != nullptr) atomicOr(a.status, SSS_FLAG_TIMEOUT);
 }
 
