@@ -317,6 +317,12 @@ __global__ void __launch_bounds__(kQThreads, 1)
     *abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  // Launched as a programmatic dependent launch: the set-up above may run
+  // while the preceding kernel drains; no global memory is touched before
+  // that kernel has completed.  The next kernel may be scheduled at once
+  // (it, in turn, waits for this one before it reads what this writes).
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   __syncthreads();
 
   if (warp == 0) {
@@ -620,8 +626,17 @@ cudaError_t quantize_launch(const float* w, const sss_qtensor_t& t, uint8_t* cli
   const int64_t nweights = t.n * t.k;
   const int64_t nchunks = (nweights + kQChunk - 1) / kQChunk;
   const int grid = static_cast<int>(std::min<int64_t>(device_sm_count(), nchunks));
-  kern<<<grid, kQThreads, kQSmem, stream>>>(w, nweights, t.codes, t.scales, t.mins, clip, status);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid), 1, 1);
+  cfg.blockDim = dim3(kQThreads, 1, 1);
+  cfg.dynamicSmemBytes = kQSmem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, w, nweights, t.codes, t.scales, t.mins, clip, status);
 }
 
 template <int Q, int GRID, int G>
