@@ -16,19 +16,26 @@
 //   warp 0     TMA producer for the fp16 activation tile (128B swizzle) and
 //              owner of the tensor-memory allocation;
 //   warp 1     a single elected thread issues tcgen05.mma (M=128, N=BN,
-//              K=16 per instruction, 4 per 64-wide k-block) and commits to
-//              the stage's "empty" barrier;
+//              K=16 per instruction, 4 per 64-wide k-block) with the weight
+//              operand A in tensor memory and the activations B in shared
+//              memory, and commits to the stage's "empty" barrier;
 //   warps 2-17 dequantise in two sets of eight that fill alternate stages:
-//              each thread owns one weight row of the tile and one 32-code
-//              half of its set's 64-wide k-blocks, loads those codes
-//              and their scale, forms fp16 s*c in natural k order and stores
-//              it with the 128B swizzle the shared-memory descriptor expects
+//              each thread owns one weight row of the tile (its tensor-memory
+//              lane) and one 32-code half of its set's 64-wide k-blocks,
+//              loads those codes and their scale, forms fp16 s*c in natural
+//              k order and writes it to the stage's A columns of tensor
+//              memory with one tcgen05.st (shared memory then carries only
+//              the activation tiles: the MMA's operand reads, the TMA writes
+//              and no generic-proxy stores)
 //              (a group whose scale lets s*c reach 65520, checked per scale
 //              as |s| 2^(q-1) or |s| (2^q - 1) + |m|, raises SSS_FLAG_RANGE);
 //              after the last k-block the same warps drain the fp32
 //              accumulator with tcgen05.ld (each set of four warps one
 //              quarter of the columns) and store Y (for a fixed token, a warp writes
 //              32 consecutive floats).
+// Tensor memory (512 columns): the fp32 accumulator in columns [0, BN), the
+// A stages in columns BN + 32 s (one 64-wide fp16 k-block of 128 rows per
+// 32 columns: lane = row, two k-consecutive halves per 32-bit column).
 // Every mbarrier wait is bounded (about one second of global time); on
 // expiry the CTA raises SSS_FLAG_TIMEOUT, all roles leave their loops, and
 // the tensor memory is still released.
@@ -101,9 +108,6 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity,
   }
 }
 
-__device__ __forceinline__ void fence_proxy_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
 __device__ __forceinline__ void tc_fence_before() {
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
@@ -147,6 +151,25 @@ __device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t a_desc, uint6
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
       "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// the same with A read from tensor memory (address a_tmem)
+__device__ __forceinline__ void umma_f16_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                            uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// 16 consecutive 32-bit columns of the warp's 32 lanes
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};\n" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15])
       : "memory");
 }
 __device__ __forceinline__ void umma_commit(uint64_t* bar) {
@@ -254,12 +277,14 @@ struct GemmArgs {
 
 template <int BN, int STAGES>
 struct Smem {
-  static constexpr int A_BYTES = kBM * kBK * 2;   // 16 KB
   static constexpr int B_BYTES = BN * kBK * 2;    // 16 or 32 KB
-  static constexpr int STAGE = A_BYTES + B_BYTES;
+  static constexpr int STAGE = B_BYTES;
   static constexpr int BAR_OFF = STAGES * STAGE;  // after the 1024-aligned stages
   static constexpr int TOTAL = BAR_OFF + (3 * STAGES + 1) * 8 + 16 + 1024;  // + align slack
+  static constexpr int A_COL = BN;                // first A-stage column in tensor memory
+  static_assert(BN + 32 * STAGES <= 512, "tensor memory holds the accumulator and A stages");
 };
+constexpr int kTmemCols = 512;
 
 template <int Q, bool ASYM, int BN, int STAGES>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -295,7 +320,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      smem_u32(tmem_slot)),
-                 "r"(BN)
+                 "r"(kTmemCols)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
@@ -312,7 +337,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int s = kb % STAGES;
         const uint32_t ph = static_cast<uint32_t>(kb / STAGES) & 1u;
         if (!mbar_wait(&empty[s], ph ^ 1u, abort)) break;
-        unsigned char* sb = smem + s * S::STAGE + S::A_BYTES;
+        unsigned char* sb = smem + s * S::STAGE;
         mbar_arrive_expect_tx(&full_b[s], S::B_BYTES);
         tma_load_2d(&xmap, &full_b[s], sb, kb * kBK, static_cast<int>(m0));
         issued = kb + 1;
@@ -334,13 +359,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait(&full_a[s], ph, abort)) break;
         if (!mbar_wait(&full_b[s], ph, abort)) break;
         tc_fence_after();
-        const uint32_t sa = smem_u32(smem + s * S::STAGE);
-        const uint32_t sb = sa + S::A_BYTES;
+        const uint32_t sb = smem_u32(smem + s * S::STAGE);
+        const uint32_t ta = tmem + static_cast<uint32_t>(S::A_COL + 32 * s);
 #pragma unroll
         for (int kk = 0; kk < kBK / 16; ++kk) {
-          // advance 16 fp16 = 32 bytes along k inside the swizzled rows
-          umma_f16(tmem, sw128_desc(sa + kk * 32), sw128_desc(sb + kk * 32), idesc,
-                   (kb | kk) != 0 ? 1u : 0u);
+          // advance 16 fp16 along k: 8 tensor-memory columns of A, 32 bytes
+          // inside the swizzled rows of B
+          umma_f16_ta(tmem, ta + 8 * kk, sw128_desc(sb + kk * 32), idesc,
+                      (kb | kk) != 0 ? 1u : 0u);
         }
         umma_commit(&empty[s]);  // frees the stage once these MMAs complete
       }
@@ -348,17 +374,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ---------------- dequantise, then epilogue ----------------
-    // thread i owns tile row (i & 127), the 32-code half hf = (i >> 7) & 1 of
-    // each 64-wide k-block, and the k-blocks kb = set, set + kDqSets, ...
-    const int i = threadIdx.x - 64;
-    const int row_i = i & (kBM - 1);
-    const int hf = (i >> 7) & 1;
-    const int set = i >> 8;
+    // a warp may touch tensor-memory lanes 32*(warp % 4) .. +31 only, so
+    // thread (warp, lane) owns tile row 32*(warp % 4) + lane; the dequant
+    // warps w = warp - 2 form four groups of four (w >> 2), each covering
+    // the 128 rows once: group g takes the 32-code half hf = g & 1 of the
+    // k-blocks kb = set, set + kDqSets, ... of set g >> 1
+    const int row_i = 32 * (warp & 3) + lane;
+    const int hf = ((warp - 2) >> 2) & 1;
+    const int set = (warp - 2) >> 3;
     const int64_t r = n0 + row_i;
     const bool rok = r < a.n;
     const int64_t nG = a.k / a.G;
     const uint8_t* rowp = a.codes + (rok ? r : 0) * (a.k * Q / 8);
-    const int sw = row_i & 7;  // swizzle phase of this row
     // codes and scale (and min) of this thread's half of one k-block
     struct KBlock {
       uint32_t w[4];
@@ -387,11 +414,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (kb >= nkb || !ok) break;
         const int s = kb % STAGES;
         const uint32_t ph = static_cast<uint32_t>(kb / STAGES) & 1u;
-        if (!mbar_wait(&empty[s], ph ^ 1u, abort)) {
+        // warp-uniform, since the tensor-memory stores below are .sync.aligned
+        const bool freed = mbar_wait(&empty[s], ph ^ 1u, abort);
+        if (!__all_sync(0xffffffffu, freed)) {
           ok = false;
           break;
         }
-        unsigned char* arow = smem + s * S::STAGE + (row_i >> 3) * 1024 + sw * 128;
+        tc_fence_after();  // the MMAs that read this stage have completed
         {
           const __half sh = __ushort_as_half(ring[q0].s);
           const __half2 s2 = __halves2half2(sh, sh);
@@ -417,14 +446,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             hv = ASYM ? __hfma2(hv, s2, m2) : __hmul2(hv, s2);    // RN16(s*c) / RN16(s*u+m)
             out[p] = *reinterpret_cast<const uint32_t*>(&hv);
           }
-#pragma unroll
-          for (int cc = 0; cc < 4; ++cc) {  // four 16-byte chunks of 8 elements
-            const int chunk = 4 * hf + cc;
-            uint4 v = make_uint4(out[4 * cc], out[4 * cc + 1], out[4 * cc + 2], out[4 * cc + 3]);
-            *reinterpret_cast<uint4*>(arow + ((chunk ^ sw) << 4)) = v;
-          }
+          // columns 16 hf .. 16 hf + 15 of stage s's A block, lane row_i
+          tmem_st16(tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16) +
+                        static_cast<uint32_t>(S::A_COL + 32 * s + 16 * hf),
+                    out);
         }
-        fence_proxy_async_smem();  // generic-proxy stores -> visible to the tensor core
+        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+        tc_fence_before();  // the stores, then the arrive the MMA issuer waits on
         __syncwarp();
         // (sss_test_set_stall: warp 2 leaves the first stage one arrive
         // short, so the MMA issuer's wait for it runs out)
@@ -437,7 +465,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------- epilogue ----------------
     // a warp may read tensor-memory lanes 32*(warp % 4) .. +31; the four
     // sets of four warps take one quarter of the columns each
-    if (ok && mbar_wait(done, 0, abort)) {
+    const bool fin = ok && mbar_wait(done, 0, abort);
+    if (__all_sync(0xffffffffu, fin)) {  // warp-uniform: tcgen05.ld is .sync.aligned
       tc_fence_after();
       const int sub = warp & 3;
       const int row_local = sub * 32 + lane;
@@ -468,7 +497,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       int drain = 0;
       (void)mbar_wait(done, 0, &drain);
     }
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(BN)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(kTmemCols)
                  : "memory");
   }
 }
@@ -509,7 +539,7 @@ size_t x16_bytes(int64_t m, int64_t k) {
 template <int Q, bool ASYM, int BN>
 cudaError_t run_gemm(const sss_qtensor_t& t, const __half* x16, int64_t m, float* y,
                      uint32_t* status, cudaStream_t stream) {
-  constexpr int STAGES = (BN == 256) ? 4 : 6;
+  constexpr int STAGES = (BN == 256) ? 6 : 8;
   using S = Smem<BN, STAGES>;
   EncodeTiledFn enc = tensor_map_encoder();
   if (enc == nullptr) return cudaErrorNotSupported;
