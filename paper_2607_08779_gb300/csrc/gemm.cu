@@ -145,21 +145,21 @@ __host__ __device__ constexpr uint32_t make_idesc(int M, int N) {
          | (static_cast<uint32_t>(M >> 4) << 24);     // M / 16
 }
 
-__device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                         uint32_t idesc, uint32_t accumulate) {
+// The four MMAs of one 64-wide k-block (K = 16 each) in one block: A from
+// tensor memory at a_tmem + 8 kk, B from the swizzled shared tile whose
+// descriptor is b_desc + 2 kk (32 bytes further along k; the start-address
+// field counts 16-byte units and does not carry), accumulating into d_tmem
+// unless first is set (the tile's first k-block starts from zero).
+__device__ __forceinline__ void umma_kblock(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                            uint32_t idesc, uint32_t first) {
   asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
-      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-// the same with A read from tensor memory (address a_tmem)
-__device__ __forceinline__ void umma_f16_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
-                                            uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      "{\n .reg .pred p;\n setp.eq.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%5], %6, %3, 1;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%7], %8, %3, 1;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%9], %10, %3, 1;\n}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(first), "r"(a_tmem + 8), "l"(b_desc + 2),
+      "r"(a_tmem + 16), "l"(b_desc + 4), "r"(a_tmem + 24), "l"(b_desc + 6)
       : "memory");
 }
 // 16 consecutive 32-bit columns of the warp's 32 lanes
@@ -275,21 +275,34 @@ struct GemmArgs {
   int stall;  // test hook: the first stage's weight tile is never announced
 };
 
-template <int BN, int STAGES>
+// Shared memory: STAGES activation tiles (1024-aligned for the 128-byte
+// swizzle), then with TW the stages' packed-code tiles (128 rows x 8q bytes)
+// and scale windows (128 rows x 8 fp16), then the barriers.
+template <int BN, int STAGES, int Q, bool TW>
 struct Smem {
-  static constexpr int B_BYTES = BN * kBK * 2;    // 16 or 32 KB
+  static constexpr int B_BYTES = BN * kBK * 2;               // 16 or 32 KB
+  static constexpr int C_BYTES = TW ? kBM * 8 * Q : 0;       // codes of one k-block
+  static constexpr int S_BYTES = TW ? kBM * 16 : 0;          // 8 scales per row
   static constexpr int STAGE = B_BYTES;
-  static constexpr int BAR_OFF = STAGES * STAGE;  // after the 1024-aligned stages
+  static constexpr int C_OFF = STAGES * B_BYTES;
+  static constexpr int S_OFF = C_OFF + STAGES * C_BYTES;
+  static constexpr int BAR_OFF = S_OFF + STAGES * S_BYTES;
   static constexpr int TOTAL = BAR_OFF + (3 * STAGES + 1) * 8 + 16 + 1024;  // + align slack
   static constexpr int A_COL = BN;                // first A-stage column in tensor memory
   static_assert(BN + 32 * STAGES <= 512, "tensor memory holds the accumulator and A stages");
+  static_assert(TOTAL <= 227 * 1024, "shared memory per CTA");
 };
 constexpr int kTmemCols = 512;
 
-template <int Q, bool ASYM, int BN, int STAGES>
+// TW: the packed codes and scales arrive by TMA with the activation tile
+// (q = 2, 4 on the symmetric grids, where a k-block's codes are 16-byte
+// aligned); otherwise each dequantising thread loads its own from global
+// memory a few k-blocks ahead.
+template <int Q, bool ASYM, int BN, int STAGES, bool TW>
 __global__ void __launch_bounds__(kThreads, 1)
-    gemm_kernel(const __grid_constant__ CUtensorMap xmap, const GemmArgs a) {
-  using S = Smem<BN, STAGES>;
+    gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap cmap,
+                const __grid_constant__ CUtensorMap smap, const GemmArgs a) {
+  using S = Smem<BN, STAGES, Q, TW>;
   extern __shared__ unsigned char smem_raw[];
   // 1024-byte alignment for the swizzle atoms
   unsigned char* smem = reinterpret_cast<unsigned char*>(
@@ -338,8 +351,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t ph = static_cast<uint32_t>(kb / STAGES) & 1u;
         if (!mbar_wait(&empty[s], ph ^ 1u, abort)) break;
         unsigned char* sb = smem + s * S::STAGE;
-        mbar_arrive_expect_tx(&full_b[s], S::B_BYTES);
+        mbar_arrive_expect_tx(&full_b[s], S::B_BYTES + S::C_BYTES + S::S_BYTES);
         tma_load_2d(&xmap, &full_b[s], sb, kb * kBK, static_cast<int>(m0));
+        if constexpr (TW) {
+          // the k-block's codes (8q bytes of each row, x a multiple of 16) and
+          // the 8-scale window holding its groups (x rounded down to 8)
+          tma_load_2d(&cmap, &full_b[s], smem + S::C_OFF + s * S::C_BYTES, kb * 8 * Q,
+                      static_cast<int>(n0));
+          tma_load_2d(&smap, &full_b[s], smem + S::S_OFF + s * S::S_BYTES,
+                      (kb * kBK / a.G) & ~7, static_cast<int>(n0));
+        }
         issued = kb + 1;
       }
       if (*abort) {
@@ -353,21 +374,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
       constexpr uint32_t idesc = make_idesc(kBM, BN);
+      // stage s: A at tensor-memory column A_COL + 32 s, B at shared offset
+      // s * STAGE (its descriptor's start-address field moves by STAGE / 16)
+      const uint32_t ta0 = tmem + static_cast<uint32_t>(S::A_COL);
+      const uint64_t bdesc0 = sw128_desc(smem_u32(smem));
+      constexpr uint64_t bstep = static_cast<uint64_t>(S::STAGE >> 4);
       for (int kb = 0; kb < nkb; ++kb) {
         const int s = kb % STAGES;
         const uint32_t ph = static_cast<uint32_t>(kb / STAGES) & 1u;
         if (!mbar_wait(&full_a[s], ph, abort)) break;
         if (!mbar_wait(&full_b[s], ph, abort)) break;
         tc_fence_after();
-        const uint32_t sb = smem_u32(smem + s * S::STAGE);
-        const uint32_t ta = tmem + static_cast<uint32_t>(S::A_COL + 32 * s);
-#pragma unroll
-        for (int kk = 0; kk < kBK / 16; ++kk) {
-          // advance 16 fp16 along k: 8 tensor-memory columns of A, 32 bytes
-          // inside the swizzled rows of B
-          umma_f16_ta(tmem, ta + 8 * kk, sw128_desc(sb + kk * 32), idesc,
-                      (kb | kk) != 0 ? 1u : 0u);
-        }
+        umma_kblock(tmem, ta0 + static_cast<uint32_t>(32 * s), bdesc0 + bstep * s, idesc,
+                    kb == 0 ? 1u : 0u);
         umma_commit(&empty[s]);  // frees the stage once these MMAs complete
       }
       umma_commit(done);
@@ -386,78 +405,119 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool rok = r < a.n;
     const int64_t nG = a.k / a.G;
     const uint8_t* rowp = a.codes + (rok ? r : 0) * (a.k * Q / 8);
-    // codes and scale (and min) of this thread's half of one k-block
-    struct KBlock {
-      uint32_t w[4];
-      uint16_t s, m;
-    };
-    auto fetch = [&](KBlock& d, int kb) {
-      if (kb >= nkb) return;
-      const int64_t kc = static_cast<int64_t>(kb) * kBK + 32 * hf;
-      const int64_t grp = kc / a.G;
-      const int sc = static_cast<int>((kc % a.G) / 32);
-      load_sub32<Q>(rowp, grp, sc, a.G, rok, d.w);
-      d.s = rok ? __ldcs(a.scales + r * nG + grp) : static_cast<uint16_t>(0);
-      if constexpr (ASYM) d.m = rok ? __ldcs(a.mins + r * nG + grp) : static_cast<uint16_t>(0);
-    };
-    // the global loads run kPrefetch of this thread's k-blocks ahead of use
-    constexpr int kPrefetch = 4;
-    KBlock ring[kPrefetch];
     bool big = false;  // a group whose s*c may leave the fp16 range
-#pragma unroll
-    for (int q0 = 0; q0 < kPrefetch; ++q0) fetch(ring[q0], set + kDqSets * q0);
     bool ok = true;
-    for (int kb0 = set; kb0 < nkb && ok; kb0 += kDqSets * kPrefetch) {
+    // fp16 s*c (ASYM: s*u + m) of the thread's 32 codes w into stage s's A
+    // columns 16 hf .. 16 hf + 15 of lane row_i, then the arrive
+    auto emit = [&](const uint32_t* w, uint16_t s16, uint16_t m16, int s, int kb) {
+      {
+        const __half sh = __ushort_as_half(s16);
+        const __half2 s2 = __halves2half2(sh, sh);
+        __half2 m2 = __float2half2_rn(0.f);
+        const float sa = fabsf(__half2float(sh));
+        if constexpr (!ASYM) big |= sa * static_cast<float>(1 << (Q - 1)) >= 65520.f;
+        if constexpr (ASYM) {
+          const __half mh = __ushort_as_half(m16);
+          m2 = __halves2half2(mh, mh);
+          big |= sa * static_cast<float>((1 << Q) - 1) + fabsf(__half2float(mh)) >= 65520.f;
+        }
+        uint32_t u[16];
+        code_pairs<Q>(w, u);
+        uint32_t out[16];
 #pragma unroll
-      for (int q0 = 0; q0 < kPrefetch; ++q0) {
-        const int kb = kb0 + kDqSets * q0;
-        if (kb >= nkb || !ok) break;
+        for (int p = 0; p < 16; ++p) {
+          // 1024 + u as fp16, minus 1024 (+ 2^(q-1) for symmetric codes): exact
+          const uint32_t mag = u[p] | 0x64006400u;
+          __half2 hv = *reinterpret_cast<const __half2*>(&mag);
+          const __half2 bias = ASYM ? __float2half2_rn(1024.f)
+                                    : __float2half2_rn(static_cast<float>(1024 + (1 << (Q - 1))));
+          hv = __hsub2(hv, bias);                               // c (or u) exactly
+          hv = ASYM ? __hfma2(hv, s2, m2) : __hmul2(hv, s2);    // RN16(s*c) / RN16(s*u+m)
+          out[p] = *reinterpret_cast<const uint32_t*>(&hv);
+        }
+        tmem_st16(tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16) +
+                      static_cast<uint32_t>(S::A_COL + 32 * s + 16 * hf),
+                  out);
+      }
+      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+      tc_fence_before();  // the stores, then the arrive the MMA issuer waits on
+      __syncwarp();
+      // (sss_test_set_stall: warp 2 leaves the first stage one arrive
+      // short, so the MMA issuer's wait for it runs out)
+      if (lane == 0 && !(a.stall && kb == 0 && warp == 2)) mbar_arrive(&full_a[s]);
+    };
+    if constexpr (TW) {
+      for (int kb = set; kb < nkb; kb += kDqSets) {
         const int s = kb % STAGES;
         const uint32_t ph = static_cast<uint32_t>(kb / STAGES) & 1u;
-        // warp-uniform, since the tensor-memory stores below are .sync.aligned
+        // warp-uniform, since the tensor-memory stores are .sync.aligned:
+        // the stage's A columns are free and its code and scale tiles landed
         const bool freed = mbar_wait(&empty[s], ph ^ 1u, abort);
         if (!__all_sync(0xffffffffu, freed)) {
           ok = false;
           break;
         }
-        tc_fence_after();  // the MMAs that read this stage have completed
-        {
-          const __half sh = __ushort_as_half(ring[q0].s);
-          const __half2 s2 = __halves2half2(sh, sh);
-          __half2 m2 = __float2half2_rn(0.f);
-          const float sa = fabsf(__half2float(sh));
-          if constexpr (!ASYM) big |= sa * static_cast<float>(1 << (Q - 1)) >= 65520.f;
-          if constexpr (ASYM) {
-            const __half mh = __ushort_as_half(ring[q0].m);
-            m2 = __halves2half2(mh, mh);
-            big |= sa * static_cast<float>((1 << Q) - 1) + fabsf(__half2float(mh)) >= 65520.f;
-          }
-          uint32_t u[16];
-          code_pairs<Q>(ring[q0].w, u);
-          uint32_t out[16];
-#pragma unroll
-          for (int p = 0; p < 16; ++p) {
-            // 1024 + u as fp16, minus 1024 (+ 2^(q-1) for symmetric codes): exact
-            const uint32_t mag = u[p] | 0x64006400u;
-            __half2 hv = *reinterpret_cast<const __half2*>(&mag);
-            const __half2 bias = ASYM ? __float2half2_rn(1024.f)
-                                      : __float2half2_rn(static_cast<float>(1024 + (1 << (Q - 1))));
-            hv = __hsub2(hv, bias);                               // c (or u) exactly
-            hv = ASYM ? __hfma2(hv, s2, m2) : __hmul2(hv, s2);    // RN16(s*c) / RN16(s*u+m)
-            out[p] = *reinterpret_cast<const uint32_t*>(&hv);
-          }
-          // columns 16 hf .. 16 hf + 15 of stage s's A block, lane row_i
-          tmem_st16(tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16) +
-                        static_cast<uint32_t>(S::A_COL + 32 * s + 16 * hf),
-                    out);
+        const bool landed = mbar_wait(&full_b[s], ph, abort);
+        if (!__all_sync(0xffffffffu, landed)) {
+          ok = false;
+          break;
         }
-        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-        tc_fence_before();  // the stores, then the arrive the MMA issuer waits on
-        __syncwarp();
-        // (sss_test_set_stall: warp 2 leaves the first stage one arrive
-        // short, so the MMA issuer's wait for it runs out)
-        if (lane == 0 && !(a.stall && kb == 0 && warp == 2)) mbar_arrive(&full_a[s]);
-        fetch(ring[q0], kb + kDqSets * kPrefetch);
+        tc_fence_after();  // the MMAs that read this stage have completed
+        const unsigned char* cs = smem + S::C_OFF + s * S::C_BYTES + row_i * (8 * Q) + hf * (4 * Q);
+        uint32_t w[4] = {0u, 0u, 0u, 0u};
+        if constexpr (Q == 4) {
+          const uint4 v = *reinterpret_cast<const uint4*>(cs);
+          w[0] = v.x; w[1] = v.y; w[2] = v.z; w[3] = v.w;
+        } else {
+          const uint2 v = *reinterpret_cast<const uint2*>(cs);
+          w[0] = v.x; w[1] = v.y;
+        }
+        const int gi = (kb * kBK + 32 * hf) / a.G, g0 = (kb * kBK / a.G) & ~7;
+        const uint16_t s16 = *reinterpret_cast<const uint16_t*>(
+            smem + S::S_OFF + s * S::S_BYTES + row_i * 16 + 2 * (gi - g0));
+        emit(w, s16, 0, s, kb);
+      }
+    } else {
+      const int64_t r = n0 + row_i;
+      const bool rok = r < a.n;
+      const int64_t nG = a.k / a.G;
+      const uint8_t* rowp = a.codes + (rok ? r : 0) * (a.k * Q / 8);
+      // codes and scale (and min) of this thread's half of one k-block
+      struct KBlock {
+        uint32_t w[4];
+        uint16_t s, m;
+      };
+      auto fetch = [&](KBlock& d, int kb) {
+        if (kb >= nkb) return;
+        const int64_t kc = static_cast<int64_t>(kb) * kBK + 32 * hf;
+        const int64_t grp = kc / a.G;
+        const int sc = static_cast<int>((kc % a.G) / 32);
+        load_sub32<Q>(rowp, grp, sc, a.G, rok, d.w);
+        d.s = rok ? __ldcs(a.scales + r * nG + grp) : static_cast<uint16_t>(0);
+        if constexpr (ASYM) d.m = rok ? __ldcs(a.mins + r * nG + grp) : static_cast<uint16_t>(0);
+      };
+      // the global loads run kPrefetch of this thread's k-blocks ahead of use
+      constexpr int kPrefetch = 4;
+      KBlock ring[kPrefetch];
+#pragma unroll
+      for (int q0 = 0; q0 < kPrefetch; ++q0) fetch(ring[q0], set + kDqSets * q0);
+      for (int kb0 = set; kb0 < nkb && ok; kb0 += kDqSets * kPrefetch) {
+#pragma unroll
+        for (int q0 = 0; q0 < kPrefetch; ++q0) {
+          const int kb = kb0 + kDqSets * q0;
+          if (kb >= nkb || !ok) break;
+          const int s = kb % STAGES;
+          const uint32_t ph = static_cast<uint32_t>(kb / STAGES) & 1u;
+          // warp-uniform, since the tensor-memory stores are .sync.aligned
+          const bool freed = mbar_wait(&empty[s], ph ^ 1u, abort);
+          if (!__all_sync(0xffffffffu, freed)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();  // the MMAs that read this stage have completed
+          emit(ring[q0].w, ring[q0].s, ring[q0].m, s, kb);
+          fetch(ring[q0], kb + kDqSets * kPrefetch);
+        }
       }
     }
     if (__any_sync(0xffffffffu, big) && lane == 0 && a.status != nullptr)
@@ -536,11 +596,11 @@ size_t x16_bytes(int64_t m, int64_t k) {
   return (mm * kk * 2 + 255) / 256 * 256;
 }
 
-template <int Q, bool ASYM, int BN>
+template <int Q, bool ASYM, int BN, bool TW>
 cudaError_t run_gemm(const sss_qtensor_t& t, const __half* x16, int64_t m, float* y,
                      uint32_t* status, cudaStream_t stream) {
-  constexpr int STAGES = (BN == 256) ? 6 : 8;
-  using S = Smem<BN, STAGES>;
+  constexpr int STAGES = (BN == 256) ? (TW ? 5 : 6) : 8;
+  using S = Smem<BN, STAGES, Q, TW>;
   EncodeTiledFn enc = tensor_map_encoder();
   if (enc == nullptr) return cudaErrorNotSupported;
   CUtensorMap map;
@@ -553,7 +613,28 @@ cudaError_t run_gemm(const sss_qtensor_t& t, const __half* x16, int64_t m, float
                     CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
-  auto kern = gemm_kernel<Q, ASYM, BN, STAGES>;
+  CUtensorMap cmap = map, smap = map;
+  if constexpr (TW) {
+    // packed codes [n][k q / 8] bytes: one k-block is 8q bytes of 128 rows;
+    // scales [n][k / G] fp16: a window of 8 (16 bytes) of 128 rows; rows
+    // past n read as zero
+    const cuuint64_t cd[2] = {static_cast<cuuint64_t>(t.k * Q / 8), static_cast<cuuint64_t>(t.n)};
+    const cuuint64_t cs[1] = {static_cast<cuuint64_t>(t.k * Q / 8)};
+    const cuuint32_t cb[2] = {static_cast<cuuint32_t>(8 * Q), kBM};
+    cr = enc(&cmap, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, t.codes, cd, cs, cb, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    const int64_t ng = t.k / t.group;
+    const cuuint64_t sd[2] = {static_cast<cuuint64_t>(ng), static_cast<cuuint64_t>(t.n)};
+    const cuuint64_t ss[1] = {static_cast<cuuint64_t>(ng * 2)};
+    const cuuint32_t sbx[2] = {8, kBM};
+    cr = enc(&smap, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, t.scales, sd, ss, sbx, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
+  }
+  auto kern = gemm_kernel<Q, ASYM, BN, STAGES, TW>;
   cudaError_t e = ensure_smem(kern, S::TOTAL);
   if (e != cudaSuccess) return e;
   GemmArgs a;
@@ -568,15 +649,31 @@ cudaError_t run_gemm(const sss_qtensor_t& t, const __half* x16, int64_t m, float
   a.G = t.group;
   a.stall = (test_stall_mask() & SSS_TEST_STALL_GEMM) ? 1 : 0;
   dim3 grid(static_cast<unsigned>((t.n + kBM - 1) / kBM), static_cast<unsigned>((m + BN - 1) / BN));
-  kern<<<grid, kThreads, S::TOTAL, stream>>>(map, a);
+  kern<<<grid, kThreads, S::TOTAL, stream>>>(map, cmap, smap, a);
   return cudaGetLastError();
+}
+
+// 256-token tiles when they still give every SM a tile (each weight tile is
+// then dequantised for twice the tokens), else 128
+template <int Q, bool ASYM, bool TW>
+cudaError_t gemm_tw(const sss_qtensor_t& t, const __half* x16, int64_t m, float* y,
+                    uint32_t* status, cudaStream_t stream) {
+  const int64_t tiles256 = ((t.n + kBM - 1) / kBM) * ((m + 255) / 256);
+  if (m > 128 && tiles256 >= device_sm_count())
+    return run_gemm<Q, ASYM, 256, TW>(t, x16, m, y, status, stream);
+  return run_gemm<Q, ASYM, 128, TW>(t, x16, m, y, status, stream);
 }
 
 template <int Q, bool ASYM>
 cudaError_t gemm_bn(const sss_qtensor_t& t, const __half* x16, int64_t m, float* y,
                     uint32_t* status, cudaStream_t stream) {
-  if (m <= 1024) return run_gemm<Q, ASYM, 128>(t, x16, m, y, status, stream);
-  return run_gemm<Q, ASYM, 256>(t, x16, m, y, status, stream);
+  if constexpr (!ASYM && Q != 3) {
+    // the code and scale tiles by TMA: 16-byte aligned scale rows
+    const bool tw = (reinterpret_cast<uintptr_t>(t.scales) % 16) == 0 &&
+                    ((t.k / t.group) * 2) % 16 == 0;
+    if (tw) return gemm_tw<Q, ASYM, true>(t, x16, m, y, status, stream);
+  }
+  return gemm_tw<Q, ASYM, false>(t, x16, m, y, status, stream);
 }
 
 template <int Q>
