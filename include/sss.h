@@ -222,7 +222,10 @@ sss_status_t sss_gemv_multi(const sss_qtensor_t* const* qts, float* const* ys,
  *   x_bf16    [in]  device bf16 [m][k], 16-byte aligned.
  *   m         [in]  0 .. 2^24 tokens.
  *   y         [out] device fp32 [m][n], 16-byte aligned, n % 4 == 0.
- *   workspace [in]  as for sss_gemv with SSS_OP_GEMM.
+ *   workspace [in]  device scratch, 16-byte aligned, of ws_bytes >= m * k * 2
+ *                   (rounded up to 256); sss_workspace_bytes(qt, m,
+ *                   SSS_OP_GEMM) bytes enable split K (see there).  Its
+ *                   contents on entry are ignored.
  *   dev_status [out] nullable; SSS_FLAG_TIMEOUT if a bounded wait expired,
  *                   SSS_FLAG_RANGE as above.
  * Errors: SSS_E_ARG, SSS_E_ALIGN, SSS_E_UNSUPPORTED, SSS_E_WORKSPACE, SSS_E_CUDA.
@@ -346,7 +349,13 @@ sss_status_t sss_sign_diagnostics(const float* w, int64_t n, int64_t k, int32_t 
 #define SSS_OP_GEMV 0
 #define SSS_OP_GEMM 1
 /* Workspace bytes sss_gemv (op SSS_OP_GEMV, m_or_batch = batch) or sss_gemm
- * (op SSS_OP_GEMM, m_or_batch = m) needs for this tensor; 0 if none. */
+ * (op SSS_OP_GEMM, m_or_batch = m) needs for this tensor; 0 if none (or an
+ * invalid tensor).  For sss_gemm this is the size that lets the call take
+ * its fastest plan: the fp16 copy of X (m * k * 2 bytes, rounded up to 256),
+ * plus, when the weight tiles are fewer than the SMs, room for fp32 partial
+ * tiles of K split across CTAs (summed in a fixed order, so the result does
+ * not depend on timing).  sss_gemm runs with any workspace that holds the
+ * fp16 copy of X, unsplit when the partials do not fit. */
 size_t sss_workspace_bytes(const sss_qtensor_t* qt, int64_t m_or_batch,
                            int32_t op);
 

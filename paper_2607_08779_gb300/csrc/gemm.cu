@@ -51,9 +51,11 @@ namespace {
 
 constexpr int kBM = 128;            // weight rows per tile (MMA M)
 constexpr int kBK = 64;             // k per stage (128 bytes of fp16)
-constexpr int kDqSets = 2;          // sets of 8 dequantising warps, on alternate k-blocks
 constexpr int kDqWarps = 8;         // warps that fill one stage
-constexpr int kThreads = 64 + 32 * kDqWarps * kDqSets;  // + producer, MMA issuer
+// threads of a CTA with SETS sets of 8 dequantising warps (on alternate
+// k-blocks), the producer warp and the MMA issuer's warp
+template <int SETS>
+constexpr int threads_of() { return 64 + 32 * kDqWarps * SETS; }
 constexpr uint64_t kWaitNs = 1000000000ull;  // bounded waits: 1 s
 
 // ---------------------------------------------------------------------------
@@ -273,6 +275,12 @@ struct GemmArgs {
   int64_t m, n, k;
   int G;
   int stall;  // test hook: the first stage's weight tile is never announced
+  // split K: CTA z of nsplit takes k-blocks [z * chunk, ...) and leaves its
+  // fp32 tile in part + z * m * n; the last of a tile's splits to finish
+  // (counted in cnt, zero on entry) sums them in split order into y
+  int nsplit;
+  float* part;
+  int* cnt;
 };
 
 // Shared memory: STAGES activation tiles (1024-aligned for the 128-byte
@@ -289,20 +297,24 @@ struct Smem {
   static constexpr int BAR_OFF = S_OFF + STAGES * S_BYTES;
   static constexpr int TOTAL = BAR_OFF + (3 * STAGES + 1) * 8 + 16 + 1024;  // + align slack
   static constexpr int A_COL = BN;                // first A-stage column in tensor memory
-  static_assert(BN + 32 * STAGES <= 512, "tensor memory holds the accumulator and A stages");
   static_assert(TOTAL <= 227 * 1024, "shared memory per CTA");
 };
-constexpr int kTmemCols = 512;
+// tensor-memory columns a CTA allocates: all 512 with one CTA per SM, half
+// when two CTAs (one dequantising set each) share an SM
+template <int SETS>
+constexpr int tmem_cols_of() { return SETS == 1 ? 256 : 512; }
 
 // TW: the packed codes and scales arrive by TMA with the activation tile
 // (q = 2, 4 on the symmetric grids, where a k-block's codes are 16-byte
 // aligned); otherwise each dequantising thread loads its own from global
 // memory a few k-blocks ahead.
-template <int Q, bool ASYM, int BN, int STAGES, bool TW>
-__global__ void __launch_bounds__(kThreads, 1)
+template <int Q, bool ASYM, int BN, int STAGES, bool TW, int SETS>
+__global__ void __launch_bounds__(threads_of<SETS>(), SETS == 1 ? 2 : 1)
     gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap cmap,
                 const __grid_constant__ CUtensorMap smap, const GemmArgs a) {
   using S = Smem<BN, STAGES, Q, TW>;
+  constexpr int kTmemCols = tmem_cols_of<SETS>();
+  static_assert(BN + 32 * STAGES <= kTmemCols, "tensor memory holds the accumulator and A stages");
   extern __shared__ unsigned char smem_raw[];
   // 1024-byte alignment for the swizzle atoms
   unsigned char* smem = reinterpret_cast<unsigned char*>(
@@ -318,7 +330,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int lane = threadIdx.x & 31;
   const int64_t n0 = static_cast<int64_t>(blockIdx.x) * kBM;
   const int64_t m0 = static_cast<int64_t>(blockIdx.y) * BN;
-  const int nkb = static_cast<int>(a.k / kBK);
+  // this split's k-blocks: global k-block kb_base + kb for kb = 0 .. nkb - 1
+  const int nkb_all = static_cast<int>(a.k / kBK);
+  const int chunk = (nkb_all + a.nsplit - 1) / a.nsplit;
+  const int kb_base = static_cast<int>(blockIdx.z) * chunk;
+  const int nkb = min(nkb_all - kb_base, chunk);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -352,14 +368,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait(&empty[s], ph ^ 1u, abort)) break;
         unsigned char* sb = smem + s * S::STAGE;
         mbar_arrive_expect_tx(&full_b[s], S::B_BYTES + S::C_BYTES + S::S_BYTES);
-        tma_load_2d(&xmap, &full_b[s], sb, kb * kBK, static_cast<int>(m0));
+        tma_load_2d(&xmap, &full_b[s], sb, (kb_base + kb) * kBK, static_cast<int>(m0));
         if constexpr (TW) {
           // the k-block's codes (8q bytes of each row, x a multiple of 16) and
           // the 8-scale window holding its groups (x rounded down to 8)
-          tma_load_2d(&cmap, &full_b[s], smem + S::C_OFF + s * S::C_BYTES, kb * 8 * Q,
-                      static_cast<int>(n0));
+          tma_load_2d(&cmap, &full_b[s], smem + S::C_OFF + s * S::C_BYTES,
+                      (kb_base + kb) * 8 * Q, static_cast<int>(n0));
           tma_load_2d(&smap, &full_b[s], smem + S::S_OFF + s * S::S_BYTES,
-                      (kb * kBK / a.G) & ~7, static_cast<int>(n0));
+                      ((kb_base + kb) * kBK / a.G) & ~7, static_cast<int>(n0));
         }
         issued = kb + 1;
       }
@@ -397,7 +413,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // thread (warp, lane) owns tile row 32*(warp % 4) + lane; the dequant
     // warps w = warp - 2 form four groups of four (w >> 2), each covering
     // the 128 rows once: group g takes the 32-code half hf = g & 1 of the
-    // k-blocks kb = set, set + kDqSets, ... of set g >> 1
+    // k-blocks kb = set, set + SETS, ... of set g >> 1
     const int row_i = 32 * (warp & 3) + lane;
     const int hf = ((warp - 2) >> 2) & 1;
     const int set = (warp - 2) >> 3;
@@ -447,7 +463,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0 && !(a.stall && kb == 0 && warp == 2)) mbar_arrive(&full_a[s]);
     };
     if constexpr (TW) {
-      for (int kb = set; kb < nkb; kb += kDqSets) {
+      for (int kb = set; kb < nkb; kb += SETS) {
         const int s = kb % STAGES;
         const uint32_t ph = static_cast<uint32_t>(kb / STAGES) & 1u;
         // warp-uniform, since the tensor-memory stores are .sync.aligned:
@@ -472,7 +488,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint2 v = *reinterpret_cast<const uint2*>(cs);
           w[0] = v.x; w[1] = v.y;
         }
-        const int gi = (kb * kBK + 32 * hf) / a.G, g0 = (kb * kBK / a.G) & ~7;
+        const int kg = kb_base + kb;
+        const int gi = (kg * kBK + 32 * hf) / a.G, g0 = (kg * kBK / a.G) & ~7;
         const uint16_t s16 = *reinterpret_cast<const uint16_t*>(
             smem + S::S_OFF + s * S::S_BYTES + row_i * 16 + 2 * (gi - g0));
         emit(w, s16, 0, s, kb);
@@ -489,7 +506,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       auto fetch = [&](KBlock& d, int kb) {
         if (kb >= nkb) return;
-        const int64_t kc = static_cast<int64_t>(kb) * kBK + 32 * hf;
+        const int64_t kc = static_cast<int64_t>(kb_base + kb) * kBK + 32 * hf;
         const int64_t grp = kc / a.G;
         const int sc = static_cast<int>((kc % a.G) / 32);
         load_sub32<Q>(rowp, grp, sc, a.G, rok, d.w);
@@ -500,11 +517,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr int kPrefetch = 4;
       KBlock ring[kPrefetch];
 #pragma unroll
-      for (int q0 = 0; q0 < kPrefetch; ++q0) fetch(ring[q0], set + kDqSets * q0);
-      for (int kb0 = set; kb0 < nkb && ok; kb0 += kDqSets * kPrefetch) {
+      for (int q0 = 0; q0 < kPrefetch; ++q0) fetch(ring[q0], set + SETS * q0);
+      for (int kb0 = set; kb0 < nkb && ok; kb0 += SETS * kPrefetch) {
 #pragma unroll
         for (int q0 = 0; q0 < kPrefetch; ++q0) {
-          const int kb = kb0 + kDqSets * q0;
+          const int kb = kb0 + SETS * q0;
           if (kb >= nkb || !ok) break;
           const int s = kb % STAGES;
           const uint32_t ph = static_cast<uint32_t>(kb / STAGES) & 1u;
@@ -516,7 +533,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           tc_fence_after();  // the MMAs that read this stage have completed
           emit(ring[q0].w, ring[q0].s, ring[q0].m, s, kb);
-          fetch(ring[q0], kb + kDqSets * kPrefetch);
+          fetch(ring[q0], kb + SETS * kPrefetch);
         }
       }
     }
@@ -531,26 +548,59 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int sub = warp & 3;
       const int row_local = sub * 32 + lane;
       const int64_t rr = n0 + row_local;
-      constexpr int kCols = BN / (kDqWarps * kDqSets / 4);
+      constexpr int kCols = BN / (kDqWarps * SETS / 4);
       const int cbeg = ((warp - 2) >> 2) * kCols;
 #pragma unroll 1
       for (int c0 = cbeg; c0 < cbeg + kCols; c0 += 32) {
         uint32_t v[32];
         tmem_ld32(tmem + (static_cast<uint32_t>(sub * 32) << 16) + c0, v);
+        // one split: y; several: this split's partial tile
+        float* dst = a.nsplit > 1 ? a.part + static_cast<int64_t>(blockIdx.z) * a.m * a.n : a.y;
         if (rr < a.n) {
 #pragma unroll
           for (int c = 0; c < 32; ++c) {
             const int64_t mm = m0 + c0 + c;
-            if (mm < a.m) a.y[mm * a.n + rr] = __uint_as_float(v[c]);
+            if (mm < a.m) dst[mm * a.n + rr] = __uint_as_float(v[c]);
           }
         }
       }
     }
   }
 
+  if (a.nsplit > 1) __threadfence();  // this CTA's partial tile, device-wide
   tc_fence_before();
   __syncthreads();
   if (*abort && threadIdx.x == 0 && a.status != nullptr) atomicOr(a.status, SSS_FLAG_TIMEOUT);
+  if (a.nsplit > 1 && !*abort) {
+    // the tile's last split to arrive sums the partials in split order
+    // (z = 0, 1, ...: the same order whichever split is last) into y and
+    // leaves the counter at zero
+    int* cnt = a.cnt + blockIdx.y * gridDim.x + blockIdx.x;
+    volatile int* last = abort + 1;
+    if (threadIdx.x == 0) *last = atomicAdd(cnt, 1) == a.nsplit - 1;
+    __syncthreads();
+    if (*last) {
+      __threadfence();
+      // 4 consecutive rows per element (n % 4 == 0, y and the partials
+      // 16-byte aligned); the loads of several elements overlap
+      constexpr int kV = kBM / 4;  // float4 per token of the tile
+      const int64_t mn = a.m * a.n;
+#pragma unroll 4
+      for (int e = threadIdx.x; e < kV * BN; e += blockDim.x) {
+        const int64_t mm = m0 + e / kV, rr = n0 + 4 * (e % kV);
+        if (mm >= a.m || rr >= a.n) continue;
+        const float4* src = reinterpret_cast<const float4*>(a.part + mm * a.n + rr);
+        float4 acc = __ldcg(src);
+        for (int z = 1; z < a.nsplit; ++z) {
+          const float4 v = __ldcg(reinterpret_cast<const float4*>(
+              reinterpret_cast<const float*>(src) + z * mn));
+          acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+        }
+        *reinterpret_cast<float4*>(a.y + mm * a.n + rr) = acc;
+      }
+      if (threadIdx.x == 0) *cnt = 0;
+    }
+  }
   if (warp == 0) {
     tc_fence_after();
     if (*abort) {  // MMAs still in flight must retire before the TMEM is released
@@ -596,9 +646,48 @@ size_t x16_bytes(int64_t m, int64_t k) {
   return (mm * kk * 2 + 255) / 256 * 256;
 }
 
-template <int Q, bool ASYM, int BN, bool TW>
+// How a call runs: tile width, dequantising sets per CTA, K splits.
+struct GemmPlan {
+  int bn, sets, nsplit;
+};
+
+// Workspace layout: fp16 X, then (split K) the partial tiles, then the
+// per-tile counters.
+size_t round256(size_t b) { return (b + 255) / 256 * 256; }
+size_t split_bytes(const sss_qtensor_t& t, int64_t m, const GemmPlan& p) {
+  if (p.nsplit <= 1) return 0;
+  const size_t tiles = static_cast<size_t>((t.n + kBM - 1) / kBM) * ((m + p.bn - 1) / p.bn);
+  return round256(static_cast<size_t>(p.nsplit) * m * t.n * 4) + round256(tiles * 4);
+}
+
+// 256-token tiles when they still give every SM a tile (each weight tile is
+// then dequantised for twice the tokens); else 128-token tiles, and when
+// those leave at least half the SMs idle, K split over as many CTAs as fill
+// them (each split at least 8 k-blocks), as far as the workspace (ws bytes)
+// holds the partial tiles.  (Two smaller CTAs per SM, one dequantising set
+// each, measured slower than one full CTA: their rings are half as deep.)
+GemmPlan plan_gemm(const sss_qtensor_t& t, int64_t m, size_t ws) {
+  const int64_t sms = device_sm_count();
+  const int64_t rt = (t.n + kBM - 1) / kBM;
+  if (m > 128 && rt * ((m + 255) / 256) >= sms) return {256, 2, 1};
+  const int64_t tiles = rt * ((m + 127) / 128);
+  if (tiles >= sms) return {128, 2, 1};
+  const int64_t nkb = t.k / kBK;
+  int split = static_cast<int>(std::min<int64_t>(sms / std::max<int64_t>(tiles, 1), nkb / 8));
+  if (split >= 2) {  // every split non-empty: as many as chunks of ceil(nkb / split)
+    const int64_t chunk = (nkb + split - 1) / split;
+    split = static_cast<int>((nkb + chunk - 1) / chunk);
+  }
+  for (; split >= 2; --split) {
+    const GemmPlan p{128, 2, split};
+    if (x16_bytes(m, t.k) <= ws && x16_bytes(m, t.k) + split_bytes(t, m, p) <= ws) return p;
+  }
+  return {128, 2, 1};
+}
+
+template <int Q, bool ASYM, int BN, bool TW, int SETS>
 cudaError_t run_gemm(const sss_qtensor_t& t, const __half* x16, int64_t m, float* y,
-                     uint32_t* status, cudaStream_t stream) {
+                     uint32_t* status, cudaStream_t stream, int nsplit, unsigned char* ws_split) {
   constexpr int STAGES = (BN == 256) ? (TW ? 5 : 6) : 8;
   using S = Smem<BN, STAGES, Q, TW>;
   EncodeTiledFn enc = tensor_map_encoder();
@@ -634,7 +723,7 @@ cudaError_t run_gemm(const sss_qtensor_t& t, const __half* x16, int64_t m, float
              CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
   }
-  auto kern = gemm_kernel<Q, ASYM, BN, STAGES, TW>;
+  auto kern = gemm_kernel<Q, ASYM, BN, STAGES, TW, SETS>;
   cudaError_t e = ensure_smem(kern, S::TOTAL);
   if (e != cudaSuccess) return e;
   GemmArgs a;
@@ -648,48 +737,68 @@ cudaError_t run_gemm(const sss_qtensor_t& t, const __half* x16, int64_t m, float
   a.k = t.k;
   a.G = t.group;
   a.stall = (test_stall_mask() & SSS_TEST_STALL_GEMM) ? 1 : 0;
-  dim3 grid(static_cast<unsigned>((t.n + kBM - 1) / kBM), static_cast<unsigned>((m + BN - 1) / BN));
-  kern<<<grid, kThreads, S::TOTAL, stream>>>(map, cmap, smap, a);
+  a.nsplit = nsplit;
+  a.part = nullptr;
+  a.cnt = nullptr;
+  const unsigned gx = static_cast<unsigned>((t.n + kBM - 1) / kBM);
+  const unsigned gy = static_cast<unsigned>((m + BN - 1) / BN);
+  if (nsplit > 1) {
+    a.part = reinterpret_cast<float*>(ws_split);
+    a.cnt = reinterpret_cast<int*>(ws_split + round256(static_cast<size_t>(nsplit) * m * t.n * 4));
+    e = cudaMemsetAsync(a.cnt, 0, sizeof(int) * gx * gy, stream);
+    if (e != cudaSuccess) return e;
+  }
+  dim3 grid(gx, gy, static_cast<unsigned>(nsplit));
+  kern<<<grid, threads_of<SETS>(), S::TOTAL, stream>>>(map, cmap, smap, a);
   return cudaGetLastError();
 }
 
-// 256-token tiles when they still give every SM a tile (each weight tile is
-// then dequantised for twice the tokens), else 128
 template <int Q, bool ASYM, bool TW>
 cudaError_t gemm_tw(const sss_qtensor_t& t, const __half* x16, int64_t m, float* y,
-                    uint32_t* status, cudaStream_t stream) {
-  const int64_t tiles256 = ((t.n + kBM - 1) / kBM) * ((m + 255) / 256);
-  if (m > 128 && tiles256 >= device_sm_count())
-    return run_gemm<Q, ASYM, 256, TW>(t, x16, m, y, status, stream);
-  return run_gemm<Q, ASYM, 128, TW>(t, x16, m, y, status, stream);
+                    uint32_t* status, cudaStream_t stream, const GemmPlan& p,
+                    unsigned char* ws_split) {
+  if (p.bn == 256) return run_gemm<Q, ASYM, 256, TW, 2>(t, x16, m, y, status, stream, 1, nullptr);
+  return run_gemm<Q, ASYM, 128, TW, 2>(t, x16, m, y, status, stream, p.nsplit, ws_split);
 }
 
 template <int Q, bool ASYM>
 cudaError_t gemm_bn(const sss_qtensor_t& t, const __half* x16, int64_t m, float* y,
-                    uint32_t* status, cudaStream_t stream) {
+                    uint32_t* status, cudaStream_t stream, const GemmPlan& p,
+                    unsigned char* ws_split) {
   if constexpr (!ASYM && Q != 3) {
     // the code and scale tiles by TMA: 16-byte aligned scale rows
     const bool tw = (reinterpret_cast<uintptr_t>(t.scales) % 16) == 0 &&
                     ((t.k / t.group) * 2) % 16 == 0;
-    if (tw) return gemm_tw<Q, ASYM, true>(t, x16, m, y, status, stream);
+    if (tw) return gemm_tw<Q, ASYM, true>(t, x16, m, y, status, stream, p, ws_split);
   }
-  return gemm_tw<Q, ASYM, false>(t, x16, m, y, status, stream);
+  return gemm_tw<Q, ASYM, false>(t, x16, m, y, status, stream, p, ws_split);
 }
 
 template <int Q>
 cudaError_t gemm_grid(const sss_qtensor_t& t, const __half* x16, int64_t m, float* y,
-                      uint32_t* status, cudaStream_t stream) {
-  if (t.grid == SSS_GRID_ASYM) return gemm_bn<Q, true>(t, x16, m, y, status, stream);
-  return gemm_bn<Q, false>(t, x16, m, y, status, stream);
+                      uint32_t* status, cudaStream_t stream, const GemmPlan& p,
+                      unsigned char* ws_split) {
+  if (t.grid == SSS_GRID_ASYM) return gemm_bn<Q, true>(t, x16, m, y, status, stream, p, ws_split);
+  return gemm_bn<Q, false>(t, x16, m, y, status, stream, p, ws_split);
 }
 
 }  // namespace
 
-size_t gemm_workspace_bytes(const sss_qtensor_t& t, int64_t m) { return x16_bytes(m, t.k); }
+// the workspace that lets the call take its preferred plan (with split K
+// where it helps); x16_bytes alone is enough to run it unsplit
+size_t gemm_workspace_bytes(const sss_qtensor_t& t, int64_t m) {
+  const size_t x = x16_bytes(m, t.k);
+  if (x == SIZE_MAX) return SIZE_MAX;
+  return x + split_bytes(t, m, plan_gemm(t, m, SIZE_MAX));
+}
+size_t gemm_workspace_min_bytes(const sss_qtensor_t& t, int64_t m) { return x16_bytes(m, t.k); }
 
 cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m, float* y,
-                        void* workspace, uint32_t* status, cudaStream_t stream, bool act_q8) {
+                        void* workspace, size_t ws_bytes, uint32_t* status, cudaStream_t stream,
+                        bool act_q8) {
   __half* x16 = static_cast<__half*>(workspace);
+  const GemmPlan plan = plan_gemm(t, m, ws_bytes);
+  unsigned char* ws_split = static_cast<unsigned char*>(workspace) + x16_bytes(m, t.k);
   cudaError_t e;
   if (act_q8) {
     e = launch_act_q8_f16(x, m, t.k, x16, status, stream);
@@ -702,9 +811,9 @@ cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m, fl
   }
   if (e != cudaSuccess) return e;
   switch (t.q) {
-    case 2: return gemm_grid<2>(t, x16, m, y, status, stream);
-    case 3: return gemm_grid<3>(t, x16, m, y, status, stream);
-    case 4: return gemm_grid<4>(t, x16, m, y, status, stream);
+    case 2: return gemm_grid<2>(t, x16, m, y, status, stream, plan, ws_split);
+    case 3: return gemm_grid<3>(t, x16, m, y, status, stream, plan, ws_split);
+    case 4: return gemm_grid<4>(t, x16, m, y, status, stream, plan, ws_split);
   }
   return cudaErrorInvalidValue;
 }

@@ -18,8 +18,8 @@ namespace {
 constexpr size_t kScratchBytes = size_t{32} << 20;  // 32 MiB: m * k * 2 bytes of fp16 X
 constexpr int kMaxDevices = 64;
 
-// Nothing in it needs to start at zero: each call writes the fp16 copy of
-// X it reads before reading it.
+// Each call writes the fp16 copy of X (and any split-K partial tiles)
+// before reading them, and zeroes the split counters it uses first.
 static __device__ __align__(256) unsigned char g_gemm_scratch[kScratchBytes];
 
 std::mutex g_mu;
@@ -57,7 +57,11 @@ sss_status_t sss_gemm_noalloc(const sss_qtensor_t* qt, const uint16_t* x_bf16, i
   // sss_gemm itself rejects m outside 0..2^24 with SSS_E_ARG; a larger m
   // must not reach the size check below as a wrapped byte count
   if (m < 0 || m > (int64_t{1} << 24)) return SSS_E_ARG;
-  const size_t need = sss_workspace_bytes(qt, m, SSS_OP_GEMM);
+  // the fp16 copy of X must fit (the call also keeps split-K partial tiles
+  // in the array when they fit beside it)
+  const size_t need = sss_workspace_bytes(qt, m, SSS_OP_GEMM) == 0
+                          ? 0
+                          : sss::gemm_workspace_min_bytes(*qt, m);
   if (need > kScratchBytes) {
     sss::set_error_message("sss_gemm_noalloc: the fp16 copy of X needs more than the "
                            "32 MiB static scratch (m * k * 2 bytes > 33554432)");

@@ -261,14 +261,16 @@ sss_status_t gemm_common(const char* name, const sss_qtensor_t* qt, const uint16
       !aligned(qt->scales, 2) || (qt->mins && !aligned(qt->mins, 2)))
     return SSS_E_ALIGN;
   if (dev_status && !aligned(dev_status, 4)) return SSS_E_ALIGN;
-  const size_t need = gemm_workspace_bytes(*qt, m);
+  // the fp16 copy of X must fit; a workspace of sss_workspace_bytes also
+  // holds the split-K partial tiles, which the call then uses where they help
+  const size_t need = gemm_workspace_min_bytes(*qt, m);
   if (need > 0 && (workspace == nullptr || ws_bytes < need)) return SSS_E_WORKSPACE;
   if (workspace != nullptr && !aligned(workspace, 16)) return SSS_E_ALIGN;
   if (qt->k == 0) {
     return finish(name, cudaMemsetAsync(y, 0, sizeof(float) * static_cast<size_t>(m) * qt->n,
                                         static_cast<cudaStream_t>(stream)));
   }
-  return finish(name, launch_gemm(*qt, x_bf16, m, y, workspace, dev_status,
+  return finish(name, launch_gemm(*qt, x_bf16, m, y, workspace, ws_bytes, dev_status,
                                   static_cast<cudaStream_t>(stream), act_q8));
 }
 }  // namespace

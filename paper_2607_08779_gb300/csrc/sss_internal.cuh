@@ -44,8 +44,9 @@ cudaError_t launch_gemv_batch(const sss_qtensor_t& t, const uint16_t* x, int bat
                               uint32_t* status, cudaStream_t stream);
 
 size_t gemm_workspace_bytes(const sss_qtensor_t& t, int64_t m);
+size_t gemm_workspace_min_bytes(const sss_qtensor_t& t, int64_t m);
 cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m,
-                        float* y, void* workspace, uint32_t* status,
+                        float* y, void* workspace, size_t ws_bytes, uint32_t* status,
                         cudaStream_t stream, bool act_q8 = false);
 
 cudaError_t launch_act_q8(const uint16_t* x, int64_t rows, int64_t k, int8_t* q, uint16_t* d,
