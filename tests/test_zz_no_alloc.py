@@ -44,7 +44,8 @@ def test_noalloc_rejects_sizes_beyond_the_scratch():
     k = 1024
     m_ok = limit // (2 * k)          # exactly fills the scratch
     qt, _ = _case(64, k, 1, 4, sss.GRID_SIGNED_SYM, 9)
-    X = torch.zeros((m_ok + 1, k), dtype=torch.bfloat16, device="cuda")
+    # seeded N(0,1) activations, so the comparison below checks real values
+    X = inputs.normal_bf16_cuda((m_ok + 1, k), 31)
     y = torch.zeros((m_ok + 1, 64), dtype=torch.float32, device="cuda")
     with pytest.raises(sss.SssError) as e:
         sss.sss_gemm_noalloc(qt, X, y)
@@ -54,4 +55,8 @@ def test_noalloc_rejects_sizes_beyond_the_scratch():
     sss.sss_gemm_noalloc(qt, X[:m_ok], y[:m_ok])
     torch.cuda.synchronize()
     ref = sss.sss_gemm(qt, X[:m_ok]).cpu().numpy()
-    assert np.array_equal(y[:m_ok].cpu().numpy(), ref)
+    got = y[:m_ok].cpu().numpy()
+    assert np.abs(ref).max() > 0
+    # the same kernel plan (no room, and no need, for split K at this shape)
+    # on the same inputs: the same bits
+    assert np.array_equal(got, ref)
