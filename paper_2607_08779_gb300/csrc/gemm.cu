@@ -660,29 +660,46 @@ size_t split_bytes(const sss_qtensor_t& t, int64_t m, const GemmPlan& p) {
   return round256(static_cast<size_t>(p.nsplit) * m * t.n * 4) + round256(tiles * 4);
 }
 
-// 256-token tiles when they still give every SM a tile (each weight tile is
-// then dequantised for twice the tokens); else 128-token tiles, and when
-// those leave at least half the SMs idle, K split over as many CTAs as fill
-// them (each split at least 8 k-blocks), as far as the workspace (ws bytes)
-// holds the partial tiles.  (Two smaller CTAs per SM, one dequantising set
-// each, measured slower than one full CTA: their rings are half as deep.)
-GemmPlan plan_gemm(const sss_qtensor_t& t, int64_t m, size_t ws) {
+// Largest K split (>= 2 to count) that fills the idle SMs with `tiles`
+// tiles, keeps every split non-empty and at least `min_kb` k-blocks long,
+// and whose partial tiles fit in the workspace (ws bytes); 1 if none.
+int split_for(const sss_qtensor_t& t, int64_t m, size_t ws, int bn, int64_t tiles,
+              int64_t min_kb) {
   const int64_t sms = device_sm_count();
-  const int64_t rt = (t.n + kBM - 1) / kBM;
-  if (m > 128 && rt * ((m + 255) / 256) >= sms) return {256, 2, 1};
-  const int64_t tiles = rt * ((m + 127) / 128);
-  if (tiles >= sms) return {128, 2, 1};
   const int64_t nkb = t.k / kBK;
-  int split = static_cast<int>(std::min<int64_t>(sms / std::max<int64_t>(tiles, 1), nkb / 8));
+  int split = static_cast<int>(std::min<int64_t>(sms / std::max<int64_t>(tiles, 1), nkb / min_kb));
   if (split >= 2) {  // every split non-empty: as many as chunks of ceil(nkb / split)
     const int64_t chunk = (nkb + split - 1) / split;
     split = static_cast<int>((nkb + chunk - 1) / chunk);
   }
   for (; split >= 2; --split) {
-    const GemmPlan p{128, 2, split};
-    if (x16_bytes(m, t.k) <= ws && x16_bytes(m, t.k) + split_bytes(t, m, p) <= ws) return p;
+    const GemmPlan p{bn, 2, split};
+    if (x16_bytes(m, t.k) <= ws && x16_bytes(m, t.k) + split_bytes(t, m, p) <= ws) return split;
   }
-  return {128, 2, 1};
+  return 1;
+}
+
+// 256-token tiles when they cover the SMs (each weight tile is then
+// dequantised for twice the tokens, and a k-block's MMAs take about as long
+// at N = 256 as at N = 128).  Otherwise, when each split keeps at least 64
+// k-blocks, 256-token tiles with K split over as many CTAs as fill the SMs;
+// else 128-token tiles, split (at least 8 k-blocks each) when they leave
+// SMs idle.  The tile's last split sums all partials alone, so a split pays
+// only with enough k-blocks behind it.  (Two half-size CTAs per SM, one
+// dequantising set each, measured slower than one full CTA: their rings are
+// half as deep.)
+GemmPlan plan_gemm(const sss_qtensor_t& t, int64_t m, size_t ws) {
+  const int64_t sms = device_sm_count();
+  const int64_t rt = (t.n + kBM - 1) / kBM;
+  if (m > 128) {
+    const int64_t tiles = rt * ((m + 255) / 256);
+    if (tiles >= sms) return {256, 2, 1};
+    const int split = split_for(t, m, ws, 256, tiles, 64);
+    if (split >= 2) return {256, 2, split};
+  }
+  const int64_t tiles = rt * ((m + 127) / 128);
+  if (tiles >= sms) return {128, 2, 1};
+  return {128, 2, split_for(t, m, ws, 128, tiles, 8)};
 }
 
 template <int Q, bool ASYM, int BN, bool TW, int SETS>
@@ -757,7 +774,8 @@ template <int Q, bool ASYM, bool TW>
 cudaError_t gemm_tw(const sss_qtensor_t& t, const __half* x16, int64_t m, float* y,
                     uint32_t* status, cudaStream_t stream, const GemmPlan& p,
                     unsigned char* ws_split) {
-  if (p.bn == 256) return run_gemm<Q, ASYM, 256, TW, 2>(t, x16, m, y, status, stream, 1, nullptr);
+  if (p.bn == 256)
+    return run_gemm<Q, ASYM, 256, TW, 2>(t, x16, m, y, status, stream, p.nsplit, ws_split);
   return run_gemm<Q, ASYM, 128, TW, 2>(t, x16, m, y, status, stream, p.nsplit, ws_split);
 }
 

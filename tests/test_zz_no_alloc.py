@@ -57,6 +57,6 @@ def test_noalloc_rejects_sizes_beyond_the_scratch():
     ref = sss.sss_gemm(qt, X[:m_ok]).cpu().numpy()
     got = y[:m_ok].cpu().numpy()
     assert np.abs(ref).max() > 0
-    # the same kernel plan (no room, and no need, for split K at this shape)
-    # on the same inputs: the same bits
-    assert np.array_equal(got, ref)
+    # the static scratch may leave no room for split-K partials where a full
+    # workspace has it, so the two may sum in different orders
+    assert rel_err_per_row(got, ref).max() <= REL_TOL
