@@ -582,21 +582,38 @@ __global__ void __launch_bounds__(threads_of<SETS>(), SETS == 1 ? 2 : 1)
     if (*last) {
       __threadfence();
       // 4 consecutive rows per element (n % 4 == 0, y and the partials
-      // 16-byte aligned); the loads of several elements overlap
+      // 16-byte aligned); eight elements per thread at a time, so every
+      // split's eight loads are in flight together
       constexpr int kV = kBM / 4;  // float4 per token of the tile
+      constexpr int kE = 8;
       const int64_t mn = a.m * a.n;
-#pragma unroll 4
-      for (int e = threadIdx.x; e < kV * BN; e += blockDim.x) {
-        const int64_t mm = m0 + e / kV, rr = n0 + 4 * (e % kV);
-        if (mm >= a.m || rr >= a.n) continue;
-        const float4* src = reinterpret_cast<const float4*>(a.part + mm * a.n + rr);
-        float4 acc = __ldcg(src);
-        for (int z = 1; z < a.nsplit; ++z) {
-          const float4 v = __ldcg(reinterpret_cast<const float4*>(
-              reinterpret_cast<const float*>(src) + z * mn));
-          acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+      for (int e0 = threadIdx.x; e0 < kV * BN; e0 += kE * blockDim.x) {
+        float4 acc[kE];
+        int64_t off[kE];
+        bool in[kE];
+#pragma unroll
+        for (int j = 0; j < kE; ++j) {
+          const int e = e0 + j * blockDim.x;
+          const int64_t mm = m0 + e / kV, rr = n0 + 4 * (e % kV);
+          in[j] = e < kV * BN && mm < a.m && rr < a.n;
+          off[j] = in[j] ? mm * a.n + rr : 0;
+          acc[j] = in[j] ? __ldcg(reinterpret_cast<const float4*>(a.part + off[j]))
+                         : make_float4(0.f, 0.f, 0.f, 0.f);
         }
-        *reinterpret_cast<float4*>(a.y + mm * a.n + rr) = acc;
+        for (int z = 1; z < a.nsplit; ++z) {
+          float4 v[kE];
+#pragma unroll
+          for (int j = 0; j < kE; ++j)
+            v[j] = in[j] ? __ldcg(reinterpret_cast<const float4*>(a.part + z * mn + off[j]))
+                         : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+          for (int j = 0; j < kE; ++j) {
+            acc[j].x += v[j].x; acc[j].y += v[j].y; acc[j].z += v[j].z; acc[j].w += v[j].w;
+          }
+        }
+#pragma unroll
+        for (int j = 0; j < kE; ++j)
+          if (in[j]) *reinterpret_cast<float4*>(a.y + off[j]) = acc[j];
       }
       if (threadIdx.x == 0) *cnt = 0;
     }
