@@ -357,6 +357,11 @@ __global__ void __launch_bounds__(threads_of<SETS>(), SETS == 1 ? 2 : 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // Launched as a programmatic dependent launch: the set-up above (barriers,
+  // tensor memory) overlaps the preceding kernel's drain; nothing in global
+  // memory is read or written before that kernel has completed.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
 
   if (warp == 0) {
     // ---------------- TMA producer: activation tiles ----------------
@@ -633,6 +638,10 @@ __global__ void __launch_bounds__(threads_of<SETS>(), SETS == 1 ? 2 : 1)
 // bf16 -> fp16 activation conversion (round to nearest even)
 __global__ void __launch_bounds__(256)
     bf16_to_f16_kernel(const uint16_t* __restrict__ x, __half* __restrict__ y, int64_t nvec) {
+  // programmatic dependent launch: start once the preceding kernel (which
+  // may still read the fp16 buffer) has completed
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec;
        i += stride) {
@@ -782,9 +791,17 @@ cudaError_t run_gemm(const sss_qtensor_t& t, const __half* x16, int64_t m, float
     e = cudaMemsetAsync(a.cnt, 0, sizeof(int) * gx * gy, stream);
     if (e != cudaSuccess) return e;
   }
-  dim3 grid(gx, gy, static_cast<unsigned>(nsplit));
-  kern<<<grid, threads_of<SETS>(), S::TOTAL, stream>>>(map, cmap, smap, a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(gx, gy, static_cast<unsigned>(nsplit));
+  cfg.blockDim = dim3(threads_of<SETS>(), 1, 1);
+  cfg.dynamicSmemBytes = S::TOTAL;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, map, cmap, smap, a);
 }
 
 template <int Q, bool ASYM, bool TW>
@@ -841,8 +858,16 @@ cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m, fl
     const int64_t nvec = m * t.k / 8;
     const int grid = static_cast<int>(std::min<int64_t>((nvec + 255) / 256,
                                                         static_cast<int64_t>(device_sm_count()) * 8));
-    bf16_to_f16_kernel<<<std::max(grid, 1), 256, 0, stream>>>(x, x16, nvec);
-    e = cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(std::max(grid, 1)), 1, 1);
+    cfg.blockDim = dim3(256, 1, 1);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, bf16_to_f16_kernel, x, x16, nvec);
   }
   if (e != cudaSuccess) return e;
   switch (t.q) {
