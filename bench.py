@@ -408,8 +408,11 @@ def measure_e2e(wl, args, ws, barrier):
 
     value: the whole step (quantize one fresh fp32 layer, the decode GEMV
     over the stack, the prefill GEMM), its GEMV bytes over its time, so that
-    it reads on the headline's scale.  gemv_only: the decode GEMV phase
-    alone, x copied in and y read back every step."""
+    it reads on the headline's scale.  The fresh layer is double-buffered:
+    step s + 1's copy runs on a copy stream while step s computes, as a
+    serving pipeline would overlap them; the small activation copies and
+    the read-backs stay on the compute stream.  gemv_only: the decode GEMV
+    phase alone, x copied in and y read back every step."""
     torch = wl.torch
     host_fresh = [f.cpu().pin_memory() for f in wl.fresh[0]]
     host_x = {k: v.cpu().pin_memory() for k, v in wl.x.items()}
@@ -421,7 +424,19 @@ def measure_e2e(wl, args, ws, barrier):
     d2h_y = nb(host_y)
     h2d = nb(host_fresh) + h2d_x + nb(host_X.values())
     d2h = d2h_y + nb(host_Y)
-    steps = max(1, min(args.steps, 5))
+    steps = max(10, min(args.steps, 20))
+    main = torch.cuda.current_stream()
+    copy = torch.cuda.Stream()
+    copied = [torch.cuda.Event(), torch.cuda.Event()]
+    used = [torch.cuda.Event(), torch.cuda.Event()]
+
+    def fresh_in(b):
+        # into buffer b once the step that last quantized it is done
+        copy.wait_event(used[b])
+        with torch.cuda.stream(copy):
+            for d, h in zip(wl.fresh[b], host_fresh):
+                d.copy_(h, non_blocking=True)
+        copied[b].record(copy)
 
     def x_in():
         for k in wl.x:
@@ -431,48 +446,56 @@ def measure_e2e(wl, args, ws, barrier):
         for h, d in zip(host_y, wl.y):
             h.copy_(d, non_blocking=True)
 
-    def one():
-        for d, h in zip(wl.fresh[0], host_fresh):
-            d.copy_(h, non_blocking=True)
-        x_in()
-        for k in wl.X:
-            wl.X[k].copy_(host_X[k], non_blocking=True)
-        wl.graphs["q0"].replay()
-        wl.graphs["v"].replay()
-        wl.graphs["m"].replay()
-        y_out()
-        for h, d in zip(host_Y, wl.Y):
-            h.copy_(d, non_blocking=True)
+    def run_steps(n):
+        for b in (0, 1):
+            used[b].record(main)
+        fresh_in(0)
+        for s in range(n):
+            b = s % 2
+            if s + 1 < n:
+                fresh_in(1 - b)
+            main.wait_event(copied[b])
+            x_in()
+            for k in wl.X:
+                wl.X[k].copy_(host_X[k], non_blocking=True)
+            wl.graphs["q%d" % b].replay()
+            used[b].record(main)
+            wl.graphs["v"].replay()
+            wl.graphs["m"].replay()
+            y_out()
+            for h, d in zip(host_Y, wl.Y):
+                h.copy_(d, non_blocking=True)
 
-    def gemv_one():
-        x_in()
-        wl.graphs["v"].replay()
-        y_out()
+    def gemv_steps(n):
+        for _ in range(n):
+            x_in()
+            wl.graphs["v"].replay()
+            y_out()
 
     def timed(fn, n):
-        fn()
+        fn(2)
         barrier()
         a = torch.cuda.Event(enable_timing=True)
         b = torch.cuda.Event(enable_timing=True)
         a.record()
-        for _ in range(n):
-            fn()
+        fn(n)
         b.record()
         barrier()
         return reduce_max([a.elapsed_time(b) / n], "cuda")[0]
 
-    ms = timed(one, steps)
-    ms_v = timed(gemv_one, max(steps, 10))
+    ms = timed(run_steps, steps)
+    ms_v = timed(gemv_steps, steps)
     return {"value": round(job_rate(wl.gemv_bytes, ws, 1, ms) / 1e9, 1), "unit": "GB/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "ms_per_step": round(ms, 4), "steps": steps,
             "scope": "whole step (quantize a fresh fp32 layer + decode GEMV over the stack + "
                      "prefill GEMM) with host copies; value = the step's GEMV bytes over its time",
-            "api": "sss_* calls captured once as CUDA graphs, replayed each step",
+            "api": "sss_* calls captured once as CUDA graphs, replayed each step; the fresh "
+                   "layer's host copy for step s+1 overlaps step s on a copy stream",
             "gemv_only": {"value": round(job_rate(wl.gemv_bytes, ws, 1, ms_v) / 1e9, 1),
                           "unit": "GB/s", "h2d_bytes_per_step": h2d_x,
                           "d2h_bytes_per_step": d2h_y, "ms_per_step": round(ms_v, 4),
-                          "steps": max(steps, 10)}}
+                          "steps": steps}}
 
 
 def oracle_gemv_rate(codes, scales, n_rows, k, q, xbits, seconds):
