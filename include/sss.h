@@ -76,8 +76,9 @@ typedef enum {
                                    sss_gemm: a group's fp16 weight operand may overflow
                                    (see those calls); their outputs may then hold
                                    inf or NaN                                         */
-#define SSS_FLAG_TIMEOUT 0x4u   /* a bounded pipeline wait (sss_gemm, or the batched
-                                   GEMV) expired; the output is incomplete            */
+#define SSS_FLAG_TIMEOUT 0x4u   /* a bounded pipeline wait of sss_gemm (or
+                                   sss_gemm_noalloc) expired; the output is
+                                   incomplete                                         */
 
 typedef enum { SSS_OUT_F32 = 0, SSS_OUT_F16 = 1, SSS_OUT_BF16 = 2 } sss_dtype_t;
 
@@ -162,8 +163,8 @@ sss_status_t sss_dequantize(const sss_qtensor_t* qt, void* out,
  *   workspace [in]  device scratch of ws_bytes >= sss_workspace_bytes(qt,
  *                   batch, SSS_OP_GEMV) bytes, 16-byte aligned, or NULL when
  *                   that size is 0.  Its contents on entry are ignored.
- *   dev_status [out] nullable; SSS_FLAG_TIMEOUT if a bounded wait expired,
- *                   SSS_FLAG_RANGE as above (batch 2..16).
+ *   dev_status [out] nullable; SSS_FLAG_RANGE as above (batch 2..16).  The
+ *                   GEMV kernels have no waits that could time out.
  * Errors: SSS_E_ARG, SSS_E_ALIGN, SSS_E_WORKSPACE, SSS_E_CUDA.
  */
 sss_status_t sss_gemv(const sss_qtensor_t* qt, const uint16_t* x_bf16,
@@ -384,19 +385,18 @@ size_t sss_gemm_noalloc_max_scratch_bytes(void);
 /*
  * sss_test_set_stall -- test hook for the bounded waits; the paper has no
  * counterpart.  While a bit below is set, every later launch of that kernel
- * family leaves one mbarrier one arrive short: the batched GEMV on the first
- * output tile's partial sums (only where a tile's k-range is split across
- * several warps), the GEMM on the first stage's weight tile.  The batch-1
- * streaming GEMV has no data-dependent waits (its warps meet only at
- * CTA-wide barriers), so its bit has no effect.  The wait on that barrier then runs out after its bound
- * (about one second), the kernel raises SSS_FLAG_TIMEOUT in dev_status,
- * lets its own copies and MMAs in flight finish, releases its tensor memory
- * and returns; its output is incomplete.  Nothing faults or hangs.
- * mask = 0 (the default) restores normal launches.  Process-wide; affects
- * launches issued (or captured) after the call on every thread.
+ * family leaves one mbarrier one arrive short: the GEMM on the first
+ * stage's weight tile.  The decode GEMV kernels (batch 1 and batched) have
+ * no data-dependent waits (their warps meet only at CTA-wide barriers), so
+ * their bits have no effect.  The wait on that barrier then runs out after
+ * its bound (about one second), the kernel raises SSS_FLAG_TIMEOUT in
+ * dev_status, lets its own copies and MMAs in flight finish, releases its
+ * tensor memory and returns; its output is incomplete.  Nothing faults or
+ * hangs.  mask = 0 (the default) restores normal launches.  Process-wide;
+ * affects launches issued (or captured) after the call on every thread.
  */
 #define SSS_TEST_STALL_GEMV 0x1u       /* gemv_stream_kernel: no waits, no effect               */
-#define SSS_TEST_STALL_GEMV_BATCH 0x2u /* gemv_batch_kernel (sss_gemv batch 2..16)             */
+#define SSS_TEST_STALL_GEMV_BATCH 0x2u /* gemv_batch_kernel: no waits, no effect                */
 #define SSS_TEST_STALL_GEMM 0x4u       /* gemm_kernel (sss_gemm, sss_gemm_noalloc)             */
 void sss_test_set_stall(uint32_t mask);
 

@@ -16,23 +16,30 @@
 //    scale lets its codes pass that bound raises SSS_FLAG_RANGE (checked per
 //    scale, conservatively: (|s| 2^(q-1), or |s| (2^q - 1) + |m|) * 16);
 //  * x is staged per K slab in shared memory in mma-B order, pre-divided by
-//    2^p, as fp16, one 8-column block per 8 batch rows (rows past the batch
-//    are zero);
+//    2^p, as fp16: 4 batch columns for batch 2..4, 8 for 5..8, 16 (two mma
+//    column blocks) for 9..16, columns past the batch zero.  Each thread
+//    loads four pieces of x before converting any, so staging costs about
+//    one load latency;
 //  * mma.sync m16n8k16: lane (g, t) feeds rows g and g+8 with codes of its
 //    own two 32-code sub-chunks of each 256-code unit (the bytes it loads,
 //    16-byte vector loads into a 2-deep register ring); the k order inside
-//    an mma is free, and B holds x of batch row g at those codes;
+//    an mma is free, and B holds x of batch row g at those codes (one
+//    16-byte shared load per two mmas);
 //  * persistent CTAs of 16 warps walk 16-row tiles; groups of KW warps share
-//    a tile and split its units, their partials meeting in shared memory
-//    behind bounded mbarrier waits.  For each K slab the CTA stages x once
-//    and runs all its tiles over it (results of later slabs are added to y
-//    by the same CTA).
+//    a tile and split its units.  With KW > 1 each warp leaves its partial
+//    of each tile in its own slot of a shared array, with no wait, and after
+//    the slab the CTA sums each tile's partials in warp order; with KW = 1 a
+//    warp writes y itself.  For each K slab the CTA stages x once and runs
+//    all its tiles over it (later slabs add to y, in the same CTA, so the
+//    result does not depend on timing).  The kernel has no data-dependent
+//    waits, only CTA-wide barriers around the staging and the sums.
 #include <cuda.h>
 
 #include <stdint.h>
 #include <string.h>
 
 #include <algorithm>
+#include <type_traits>
 
 #include "gemv_common.cuh"
 
@@ -56,7 +63,7 @@ struct BatchArgs {
   int64_t ntiles;
   int lgkw;        // log2(warps per tile)
   int slab_units;  // units of 256 codes per x slab
-  int stall;       // test hook: the first tile's barrier stays one arrive short
+  int rounds;      // tiles per warp group at most (the partial array's depth)
   uint32_t* status;
 };
 
@@ -96,14 +103,27 @@ __device__ __forceinline__ uint32_t magic_pair(const uint32_t* w, int p) {
   return unpack_pair<Q>(w, p) | 0x64006400u;
 }
 
-template <int Q, bool ASYM, int G, int NBLK>
+// NBC = batch columns of the staged x: 4 (batch 2..4), 8 (5..8) or 16
+// (9..16).  An mma covers 8 columns; with NBC = 4 only lanes 0..15 (columns
+// 0..3) have entries of their own, and lanes 16..31 read those of lane - 16,
+// so columns 4..7 repeat columns 0..3 and their results are dropped.
+template <int NBC>
+struct XShape {
+  static constexpr int NBLK = NBC < 8 ? 1 : NBC / 8;  // mma column blocks
+  static constexpr int LS = NBC < 8 ? 16 : 32;        // lanes with entries per block
+  static constexpr int XU = 8 * NBLK * LS * 16;       // staged x bytes per unit
+};
+
+template <int Q, bool ASYM, int G, int NBC, int D>
 __global__ void __launch_bounds__(kThreads, 1) gemv_batch_kernel(const __grid_constant__ BatchArgs a) {
-  constexpr int NBC = 8 * NBLK;             // batch columns (padded)
+  using XS = XShape<NBC>;
+  constexpr int NBLK = XS::NBLK;
+  constexpr int LS = XS::LS;
+  constexpr int XU = XS::XU;
   constexpr int R = 16;
   constexpr int HALF = 1 << (Q - 1);
   constexpr int UB = 32 * Q;                // code bytes of one row in one unit
   constexpr int SPU = 256 / G;              // scales of one row in one unit
-  constexpr int XU = 16 * 4 * NBC * 8;      // staged x bytes per unit
   extern __shared__ __align__(128) unsigned char smem[];
 
   const int nunits = static_cast<int>(a.k / 256);
@@ -115,26 +135,29 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_batch_kernel(const __grid_co
   const int SK = a.slab_units;
   const int nslabs = (nunits + SK - 1) / SK;
 
-  // ---- shared memory: x slab | partials | barriers | flag ----
-  unsigned char* xs = smem;                                      // [SK][16][NBLK][32 lanes] x 8 B
-  float* part = reinterpret_cast<float*>(xs + static_cast<size_t>(SK) * XU);  // [ngrp][2][KW][R][NBC]
-  uint64_t* pready = reinterpret_cast<uint64_t*>(part + 2 * kWarps * R * NBC);  // [kWarps][2]
-  uint64_t* pfree = pready + 2 * kWarps;
-  volatile int* abort = reinterpret_cast<volatile int*>(pfree + 2 * kWarps);
+  // ---- shared memory: x slab [SK][8][NBLK][LS] x 16 B | row partials
+  // [ngrp][rounds][KW][NBC][R] fp32 (KW > 1) ----
+  unsigned char* xs = smem;
+  float* part = reinterpret_cast<float*>(xs + static_cast<size_t>(SK) * XU);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int gq = lane >> 2, tq = lane & 3;
   const int grp = warp >> lgkw;
   const int kw = warp & (KW - 1);
+  const uint32_t xs_a = su32(xs);
 
-  if (threadIdx.x == 0) {
-    for (int i = 0; i < 2 * kWarps; ++i) {
-      bar_init(&pready[i], KW);  // every warp of a group, after its lanes wrote
-      bar_init(&pfree[i], 1);
+  // Entries of batch columns past the batch are zero (staging never writes
+  // them); this touches nothing produced upstream, so it precedes the
+  // grid-dependency wait.
+  if (a.batch < NBC) {
+    const int entries = SK * 8 * NBLK * LS;
+    for (int e = threadIdx.x; e < entries; e += kThreads) {
+      const int col = 8 * ((e / LS) % NBLK) + ((e % LS) >> 2);
+      if (col >= a.batch)
+        asm volatile("st.shared.v4.u32 [%0], {%1,%1,%1,%1};" ::"r"(xs_a + 16u * e), "r"(0u)
+                     : "memory");
     }
-    *abort = 0;
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
@@ -239,51 +262,59 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_batch_kernel(const __grid_co
   int total = 0;
   for (int s = 0; s < nslabs; ++s) total += static_cast<int>(my_tiles) * units_in(s);
 
-  Regs r0, r1;
-  set_fetch();
-  if (total > 0) fetch(r0);
-  if (total > 1) fetch(r1);
-  asm volatile("griddepcontrol.wait;" ::: "memory");  // x is produced upstream
-
-  const uint32_t xs_a = su32(xs);
-  bool ok = true;
   float acc[NBLK][4];
 #pragma unroll
   for (int nb = 0; nb < NBLK; ++nb)
 #pragma unroll
     for (int e = 0; e < 4; ++e) acc[nb][e] = 0.f;
 
-  // Stage slab s: x[b][32*(8u + sc) + e] for the slab's units u, in mma-B
-  // order: the 8 bytes at (u, j, nb, lane = 4g + t) hold, for batch column
-  // n = 8nb + g, the activation pairs 2j and 2j+1 of quad t (quad t's
-  // sub-chunk 2t + (j >> 3), pairs (2j) & 15 and (2j+1) & 15), each element
-  // pre-divided by 2^p; a warp's B fragments of one mma are then 256
-  // contiguous bytes.  One thread handles 16 elements (half a sub-chunk) of
-  // one batch row.
-  auto stage = [&](int s) {
-    const int u0 = s * SK;
-    const int su = min(SK, nunits - u0);
-    const int items = su * 8 * NBC * 2;
-    for (int it = threadIdx.x; it < items; it += kThreads) {
-      const int hf = it & 1;
-      const int n = (it >> 1) % NBC;
-      const int scu = (it >> 1) / NBC;  // sub-chunk within the slab
-      const int ul = scu >> 3, sc = scu & 7;
-      uint32_t pr[8];
-      if (n < a.batch) {
+  // Stage slab s: x[n][32*(8u + sc) + e] for the slab's units u, in mma-B
+  // order: the 16 bytes at (u, j2, nb, lane = 4g + t) hold, for batch
+  // column n = 8nb + g, the activation pairs 4j2 .. 4j2+3 of quad t (quad
+  // t's sub-chunk 2t + (j2 >> 2), pairs (4j2) & 15 .. (4j2+3) & 15), each
+  // element pre-divided by 2^p: the B operands of two consecutive mmas.  One
+  // item is 16 elements (half a sub-chunk) of one batch row; consecutive
+  // items run along k, and a thread loads U items before converting any of
+  // them, so their loads are in flight together (U = 4 for the first slab,
+  // staged before the weight ring fills; 2 for later slabs, while the
+  // ring's registers are live).
+  auto slab_items = [&](int s) { return min(SK, nunits - s * SK) * 16 * a.batch; };
+  auto stage_load = [&](int s, int base, auto& v) {
+    constexpr int U = sizeof(v) / sizeof(v[0]);
+    const int items = slab_items(s), per_row = items / a.batch;
+#pragma unroll
+    for (int c = 0; c < U; ++c) {
+      const int it = base + c * kThreads;
+      if (it < items) {
+        const int n = it / per_row, w = it - n * per_row;  // w = 2 * sub-chunk + half
         const uint4* src = reinterpret_cast<const uint4*>(
-            a.x + static_cast<int64_t>(n) * a.k + static_cast<int64_t>(u0 + ul) * 256 + 32 * sc + 16 * hf);
+            a.x + static_cast<int64_t>(n) * a.k + static_cast<int64_t>(s) * SK * 256 + 16 * w);
+        v[c][0] = __ldg(src);
+        v[c][1] = __ldg(src + 1);
+      }
+    }
+  };
+  auto stage_put = [&](int s, int base, const auto& v) {
+    constexpr int U = sizeof(v) / sizeof(v[0]);
+    const int items = slab_items(s), per_row = items / a.batch;
+#pragma unroll
+    for (int c = 0; c < U; ++c) {
+      const int it = base + c * kThreads;
+      if (it < items) {
+        const int n = it / per_row, w = it - n * per_row;
+        const int hf = w & 1, scu = w >> 1;
+        const int ul = scu >> 3, sc = scu & 7;
         float xv[16];
 #pragma unroll
-        for (int c = 0; c < 2; ++c) {
-          const uint4 v = __ldg(src + c);
-          const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
+        for (int cc = 0; cc < 2; ++cc) {
+          const uint32_t wv[4] = {v[c][cc].x, v[c][cc].y, v[c][cc].z, v[c][cc].w};
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
-            xv[8 * c + 2 * e] = __uint_as_float(wv[e] << 16);
-            xv[8 * c + 2 * e + 1] = __uint_as_float(wv[e] & 0xFFFF0000u);
+            xv[8 * cc + 2 * e] = __uint_as_float(wv[e] << 16);
+            xv[8 * cc + 2 * e + 1] = __uint_as_float(wv[e] & 0xFFFF0000u);
           }
         }
+        uint32_t pr[8];
 #pragma unroll
         for (int jj = 0; jj < 8; ++jj) {
           int ea, eb;
@@ -292,23 +323,44 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_batch_kernel(const __grid_co
           __half2 hv = __floats2half2_rn(xv[ea] * mult, xv[eb] * mult);
           pr[jj] = *reinterpret_cast<uint32_t*>(&hv);
         }
-      } else {
+        // pair P = 8hf + jj of sub-chunk sc = 2t + h is quad t's pair
+        // 16h + P: entry j2 = 4h + 2hf + (jj >> 2), 8-byte slot (jj >> 1) & 1
+        const int t = sc >> 1, h = sc & 1;
 #pragma unroll
-        for (int jj = 0; jj < 8; ++jj) pr[jj] = 0u;
-      }
-      // pair p = 8hf + jj of sub-chunk sc = 2t + h is quad t's pair
-      // P = 16h + p, i.e. entry j = P >> 1, slot P & 1
-      const int t = sc >> 1, h = sc & 1;
-#pragma unroll
-      for (int jj = 0; jj < 8; jj += 2) {
-        const int j = 8 * h + 4 * hf + (jj >> 1);
-        const uint32_t dst = xs_a + static_cast<uint32_t>(
-            ul * XU + ((j * NBLK + (n >> 3)) * 32 + 4 * (n & 7) + t) * 8);
-        asm volatile("st.shared.v2.u32 [%0], {%1,%2};" ::"r"(dst), "r"(pr[jj]), "r"(pr[jj + 1])
-                     : "memory");
+        for (int qd = 0; qd < 2; ++qd) {
+          const int j2 = 4 * h + 2 * hf + qd;
+          const uint32_t dst = xs_a + static_cast<uint32_t>(
+              ul * XU + ((j2 * NBLK + (n >> 3)) * LS + 4 * (n & 7) + t) * 16);
+          asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(dst), "r"(pr[4 * qd]),
+                       "r"(pr[4 * qd + 1]), "r"(pr[4 * qd + 2]), "r"(pr[4 * qd + 3])
+                       : "memory");
+        }
       }
     }
   };
+  auto stage_from = [&](auto u_tag, int s, int start) {
+    constexpr int U = decltype(u_tag)::value;
+    for (int base = start; base < slab_items(s); base += U * kThreads) {
+      uint4 v[U][2];
+      stage_load(s, base, v);
+      stage_put(s, base, v);
+    }
+  };
+
+  // Every global access follows the grid-dependency wait.  Slab 0 of x is
+  // staged before the weight ring is filled: its loads return from L2 in
+  // well under a microsecond, but the shared-memory stores of its
+  // conversion would otherwise wait behind the ring's DRAM loads in the
+  // SM's load/store queue.  The barrier comes before the ring's loads too,
+  // so no warp waits for another warp's loads to be issued.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  stage_from(std::integral_constant<int, 4>{}, 0, threadIdx.x);
+  __syncthreads();
+  Regs ring[D];
+  set_fetch();
+#pragma unroll
+  for (int d = 0; d < D; ++d)
+    if (d < total) fetch(ring[d]);
 
   // constants of the operand formation
   uint32_t off[3];
@@ -320,10 +372,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_batch_kernel(const __grid_co
     off[i] = *reinterpret_cast<uint32_t*>(&hv);
   }
 
-  // a group of this thread's whose operand may leave the fp16 range
+  // fp16 range of the operand: symmetric grids keep the largest |s| bit
+  // pattern of each half (fp16 magnitudes order as their bits), the min-max
+  // grid tests each group
+  uint32_t smax = 0u;
   bool big = false;
+  const uint32_t xlane = static_cast<uint32_t>(lane & (LS - 1)) * 16u;
   auto compute = [&](const Regs& rg, int ul) {
-    const uint32_t xu = xs_a + static_cast<uint32_t>(ul * XU);
+    const uint32_t xu = xs_a + static_cast<uint32_t>(ul * XU) + xlane;
+    if constexpr (!ASYM) smax = __vmaxu2(smax, __vmaxu2(rg.s[0] & 0x7FFF7FFFu, rg.s[1] & 0x7FFF7FFFu));
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
       // the fp16 scale (and min) of sub-chunk 2tq + h for rows gq, gq + 8
@@ -332,9 +389,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_batch_kernel(const __grid_co
       for (int hh = 0; hh < 2; ++hh) {
         const uint32_t sb = G == 32 ? ((rg.s[hh] >> (16 * h)) & 0xFFFFu) : (rg.s[hh] & 0xFFFFu);
         S[hh] = f16x2_of(sb);
-        const float sa = fabsf(__half2float(__ushort_as_half(static_cast<unsigned short>(sb))));
-        if constexpr (!ASYM) big |= sa * static_cast<float>(HALF * 16) >= 65520.f;
         if constexpr (ASYM) {
+          const float sa = fabsf(__half2float(__ushort_as_half(static_cast<unsigned short>(sb))));
           const uint32_t mb = G == 32 ? ((rg.m[hh] >> (16 * h)) & 0xFFFFu) : (rg.m[hh] & 0xFFFFu);
           const float ma = fabsf(__half2float(__ushort_as_half(static_cast<unsigned short>(mb))));
           big |= (sa * static_cast<float>(2 * HALF - 1) + ma) * 16.f >= 65520.f;
@@ -349,31 +405,36 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_batch_kernel(const __grid_co
         else return hmul2(t, S[hh]);
       };
 #pragma unroll
-      for (int jm = 0; jm < 8; ++jm) {
-        const int p = 2 * jm;
-        const int j = 8 * h + jm;
-        const uint32_t a0 = deq(0, p), a1 = deq(1, p), a2 = deq(0, p + 1), a3 = deq(1, p + 1);
+      for (int jm = 0; jm < 8; jm += 2) {
+        uint4 bv[NBLK];
 #pragma unroll
-        for (int nb = 0; nb < NBLK; ++nb) {
-          const float2 bv = lds64f(xu + static_cast<uint32_t>(((j * NBLK + nb) * 32 + lane) * 8));
-          mma16816(acc[nb], a0, a1, a2, a3, __float_as_uint(bv.x), __float_as_uint(bv.y));
+        for (int nb = 0; nb < NBLK; ++nb)
+          bv[nb] = lds128(xu + static_cast<uint32_t>((((4 * h + (jm >> 1)) * NBLK + nb) * LS) * 16));
+#pragma unroll
+        for (int jj = 0; jj < 2; ++jj) {
+          const int p = 2 * (jm + jj);
+          const uint32_t a0 = deq(0, p), a1 = deq(1, p), a2 = deq(0, p + 1), a3 = deq(1, p + 1);
+#pragma unroll
+          for (int nb = 0; nb < NBLK; ++nb)
+            mma16816(acc[nb], a0, a1, a2, a3, jj ? bv[nb].z : bv[nb].x, jj ? bv[nb].w : bv[nb].y);
         }
       }
     }
   };
 
-  // ---- tile end: the group's KW partials meet; y = sum (first slab) or
-  // y += sum (later slabs) ----
+  // ---- tile end: y = sum (first slab) or y += sum (later slabs).  KW = 1:
+  // the warp owns the tile and writes y itself; KW > 1: the warp leaves its
+  // partial in its own slot, summed after the slab ----
   auto tile_end = [&](int s, int64_t i) {
-    const int64_t row0 = (tfirst + i * tstride) * R;
     if (KW == 1) {
+      const int64_t row0 = (tfirst + i * tstride) * R;
 #pragma unroll
       for (int nb = 0; nb < NBLK; ++nb)
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const int64_t r = row0 + gq + 8 * (e >> 1);
           const int b = 8 * nb + 2 * tq + (e & 1);
-          if (r < a.n && b < a.batch && ok) {
+          if (r < a.n && b < a.batch) {
             float* yp = a.y + static_cast<int64_t>(b) * a.n + r;
             *yp = (s == 0 ? 0.f : *yp) + acc[nb][e];
           }
@@ -381,103 +442,132 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_batch_kernel(const __grid_co
         }
       return;
     }
-    const int bsel = static_cast<int>(i & 1);
-    // the group's tiles alternate between two partial buffers; a buffer's
-    // use count runs on over the slabs (each slab visits every tile once)
-    const int64_t per_slab = bsel == 0 ? (my_tiles + 1) >> 1 : my_tiles >> 1;
-    const uint32_t use = static_cast<uint32_t>(static_cast<int64_t>(s) * per_slab + (i >> 1)) & 1u;
-    float* pb = part + (static_cast<size_t>(grp) * 2 + bsel) * KW * R * NBC;
-    uint64_t* rdy = &pready[grp * 2 + bsel];
-    uint64_t* fre = &pfree[grp * 2 + bsel];
-    if (!bar_wait(fre, use ^ 1u, abort)) ok = false;
+    float* pb = part + ((static_cast<size_t>(grp) * a.rounds + i) * KW + kw) * (NBC * R);
 #pragma unroll
     for (int nb = 0; nb < NBLK; ++nb)
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
-        pb[(kw * R + gq + 8 * (e >> 1)) * NBC + 8 * nb + 2 * tq + (e & 1)] = acc[nb][e];
+        const int b = 8 * nb + 2 * tq + (e & 1);
+        if (b < NBC) pb[b * R + gq + 8 * (e >> 1)] = acc[nb][e];
         acc[nb][e] = 0.f;
       }
-    __syncwarp();
-    // (sss_test_set_stall: the last warp leaves the first tile's barrier one
-    // arrive short, so its reducer's wait runs out)
-    if (lane == 0 && !(a.stall && s == 0 && i == 0 && kw == KW - 1)) bar_arrive(rdy);
-    if (kw == static_cast<int>(i & (KW - 1))) {
-      if (!bar_wait(rdy, use, abort)) ok = false;
-      for (int v = lane; v < R * NBC; v += 32) {
-        const int rr = v / NBC, b = v % NBC;
-        float sum = 0.f;
-        for (int c = 0; c < KW; ++c) sum += pb[(c * R + rr) * NBC + b];
-        const int64_t r = row0 + rr;
-        if (r < a.n && b < a.batch && ok) {
-          float* yp = a.y + static_cast<int64_t>(b) * a.n + r;
-          *yp = (s == 0 ? 0.f : *yp) + sum;
-        }
-      }
-      __syncwarp();
-      if (lane == 0) bar_arrive(fre);
+  };
+  // the slab's sums of every tile's KW partials, in warp order (warps with
+  // no unit in the slab left no partial)
+  auto slab_sums = [&](int s) {
+    const int kwn = min(KW, min(SK, nunits - s * SK));
+    const int per_grp = a.rounds * NBC * R;
+    for (int idx = threadIdx.x; idx < ngrp * per_grp; idx += kThreads) {
+      const int g = idx / per_grp, rem = idx - g * per_grp;
+      const int i = rem / (NBC * R), b = (rem / R) % NBC, row = rem % R;
+      if (b >= a.batch) continue;
+      const int64_t t = (static_cast<int64_t>(i) * ngrp + g) * gridDim.x + blockIdx.x;
+      if (t >= a.ntiles) continue;
+      const int64_t r = t * R + row;
+      if (r >= a.n) continue;
+      const float* pb = part + (static_cast<size_t>(g) * a.rounds + i) * KW * (NBC * R) + b * R + row;
+      float sum = 0.f;
+      for (int c = 0; c < kwn; ++c) sum += pb[c * (NBC * R)];
+      float* yp = a.y + static_cast<int64_t>(b) * a.n + r;
+      *yp = (s == 0 ? 0.f : *yp) + sum;
     }
   };
 
-  int gk = 0;  // position in this warp's unit stream (register ring slot gk & 1)
+  // the units: unit gk of this warp's stream is computed from ring slot
+  // gk % D, which then takes unit gk + D (the switch keeps every slot's
+  // index a compile-time constant, so the ring stays in registers)
+  int gk = 0, slot = 0;
+  auto step = [&](Regs& rg, int ul) {
+    compute(rg, ul);
+    if (gk + D < total) fetch(rg);
+  };
   for (int s = 0; s < nslabs; ++s) {
-    __syncthreads();  // barriers initialised / every warp done with the previous slab
-    stage(s);
-    __syncthreads();
+    if (s > 0) {
+      __syncthreads();  // every warp done with the previous slab and its sums
+      stage_from(std::integral_constant<int, 2>{}, s, threadIdx.x);
+      __syncthreads();
+    }
     const int ups = units_in(s);
     for (int64_t i = 0; i < my_tiles; ++i) {
       for (int r = 0; r < ups; ++r, ++gk) {
         const int ul = kw + r * KW;  // unit within the slab
-        if (gk & 1) {
-          compute(r1, ul);
-          if (gk + 2 < total) fetch(r1);
-        } else {
-          compute(r0, ul);
-          if (gk + 2 < total) fetch(r0);
+        switch (slot) {
+          case 0: step(ring[0], ul); break;
+          case 1: if constexpr (D > 1) step(ring[1], ul); break;
+          case 2: if constexpr (D > 2) step(ring[2], ul); break;
+          default: if constexpr (D > 3) step(ring[3], ul); break;
         }
+        slot = slot + 1 == D ? 0 : slot + 1;
       }
       tile_end(s, i);
     }
+    if (KW > 1) {
+      __syncthreads();
+      slab_sums(s);
+    }
+  }
+  if constexpr (!ASYM) {
+    // |s| * 2^(q-1) * 16 >= 65520 exactly when |s| >= the fp16 value that
+    // 4095 / 2^(q-1) rounds up to
+    const uint32_t m = max(smax & 0xFFFFu, smax >> 16);
+    big = m >= static_cast<uint32_t>(__half_as_ushort(__float2half_ru(4095.f / HALF)));
   }
   if (__any_sync(0xffffffffu, big) && lane == 0 && a.status != nullptr)
     atomicOr(a.status, SSS_FLAG_RANGE);
-  if (*abort && threadIdx.x == 0 && a.status != nullptr) atomicOr(a.status, SSS_FLAG_TIMEOUT);
 }
 
-template <int NBLK>
-size_t batch_smem(int slab_units) {
-  return static_cast<size_t>(slab_units) * (16 * 4 * 8 * NBLK * 8) +
-         static_cast<size_t>(2 * kWarps * 16 * 8 * NBLK) * 4 + 8 * 4 * kWarps + 16;
+// Register ring depth: units of weights in flight per warp.  Two: with
+// three the unit loop, bound by instruction issue, ran no faster and the
+// first loads took longer to issue.
+constexpr int ring_depth(int, bool, int) { return 2; }
+
+template <int NBC>
+size_t batch_smem(int slab_units, int kw, int ngrp, int rounds) {
+  return static_cast<size_t>(slab_units) * XShape<NBC>::XU +
+         (kw > 1 ? static_cast<size_t>(ngrp) * rounds * kw * NBC * 16 * 4 : 0);
 }
 
-template <int Q, bool ASYM, int G, int NBLK>
+template <int Q, bool ASYM, int G, int NBC>
 cudaError_t launch_b(const sss_qtensor_t& t, BatchArgs& a, cudaStream_t stream) {
   const int nunits = static_cast<int>(t.k / 256);
-  int sk = nunits;
-  while (sk > 1 && batch_smem<NBLK>(sk) > static_cast<size_t>(kSmemMax)) sk = (sk + 1) / 2;
-  if (batch_smem<NBLK>(sk) > static_cast<size_t>(kSmemMax)) return cudaErrorNotSupported;
-  a.slab_units = sk;
-  const size_t smem = batch_smem<NBLK>(sk);
-  auto kern = gemv_batch_kernel<Q, ASYM, G, NBLK>;
-  cudaError_t e = ensure_smem(kern, static_cast<int>(smem));
-  if (e != cudaSuccess) return e;
   const int64_t tiles = (t.n + 15) / 16;
   a.ntiles = tiles;
   const int sms = device_sm_count();
   const int grid = static_cast<int>(std::min<int64_t>(sms, tiles));
   const int64_t per_cta = (tiles + grid - 1) / grid;
-  int best = 0;
+  // Warps per tile KW and slab size: minimise the busiest warp's units
+  // (rounds of the CTA's tiles x that warp's units over the slabs) plus two
+  // units' worth per extra slab (a CTA-wide barrier and a re-stage of x),
+  // preferring fewer warps per tile on ties; the slab is the largest that
+  // fits beside the partial array.
+  int best = -1, best_sk = 0;
   int64_t best_cost = INT64_MAX;
   for (int lg = 0; (1 << lg) <= kWarps; ++lg) {
     const int kwn = 1 << lg;
-    if (kwn > 1 && kwn > std::min(nunits, sk)) break;
-    const int64_t ngrp = kWarps >> lg;
-    const int64_t cost = ((per_cta + ngrp - 1) / ngrp) * ((nunits + kwn - 1) / kwn);
+    if (kwn > 1 && kwn > nunits) break;
+    const int ngrp = kWarps >> lg;
+    const int64_t rounds = (per_cta + ngrp - 1) / ngrp;
+    const size_t parts = batch_smem<NBC>(0, kwn, ngrp, static_cast<int>(std::min<int64_t>(rounds, 1 << 20)));
+    if (parts + XShape<NBC>::XU > static_cast<size_t>(kSmemMax)) continue;
+    const int sk = static_cast<int>(std::min<size_t>(nunits, (kSmemMax - parts) / XShape<NBC>::XU));
+    const int nslabs = (nunits + sk - 1) / sk;
+    int64_t units = 0;
+    for (int s = 0; s < nslabs; ++s) units += (std::min(sk, nunits - s * sk) + kwn - 1) / kwn;
+    const int64_t cost = rounds * units + 2 * (nslabs - 1);
     if (cost < best_cost) {
       best_cost = cost;
       best = lg;
+      best_sk = sk;
     }
   }
+  if (best < 0) return cudaErrorNotSupported;
   a.lgkw = best;
+  a.slab_units = best_sk;
+  a.rounds = static_cast<int>((per_cta + (kWarps >> best) - 1) / (kWarps >> best));
+  const size_t smem = batch_smem<NBC>(best_sk, 1 << best, kWarps >> best, a.rounds);
+  auto kern = gemv_batch_kernel<Q, ASYM, G, NBC, ring_depth(Q, ASYM, NBC)>;
+  cudaError_t e = ensure_smem(kern, static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(grid), 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
@@ -488,7 +578,9 @@ cudaError_t launch_b(const sss_qtensor_t& t, BatchArgs& a, cudaStream_t stream) 
 
 template <int Q, bool ASYM, int G>
 cudaError_t launch_bn(const sss_qtensor_t& t, BatchArgs& a, cudaStream_t stream) {
-  return a.batch <= 8 ? launch_b<Q, ASYM, G, 1>(t, a, stream) : launch_b<Q, ASYM, G, 2>(t, a, stream);
+  if (a.batch <= 4) return launch_b<Q, ASYM, G, 4>(t, a, stream);
+  if (a.batch <= 8) return launch_b<Q, ASYM, G, 8>(t, a, stream);
+  return launch_b<Q, ASYM, G, 16>(t, a, stream);
 }
 
 template <int Q, bool ASYM>
@@ -528,7 +620,6 @@ cudaError_t launch_gemv_batch(const sss_qtensor_t& t, const uint16_t* x, int bat
   a.k = t.k;
   a.batch = batch;
   a.status = status;
-  a.stall = (test_stall_mask() & SSS_TEST_STALL_GEMV_BATCH) ? 1 : 0;
   const bool asym = t.grid == SSS_GRID_ASYM;
   switch (t.q) {
     case 2: return asym ? launch_bg<2, true>(t, a, stream) : launch_bg<2, false>(t, a, stream);

@@ -1,7 +1,7 @@
 // gemv_common.cuh -- pieces shared by the decode GEMV kernels
-// (gemv_stream.cu, gemv_batch.cu): bounded mbarrier waits, mma.sync
-// m16n8k16 wrappers, shared-memory loads, and the code-pair unpack of the
-// batched kernel (fields at bit 0, 2 or 4 of each fp16 half).
+// (gemv_stream.cu, gemv_batch.cu): mma.sync m16n8k16 wrappers,
+// shared-memory loads, and the code-pair unpack of the batched kernel
+// (fields at bit 0, 2 or 4 of each fp16 half).
 #pragma once
 
 #include <stdint.h>
@@ -11,8 +11,6 @@
 namespace sss {
 namespace gv {
 
-constexpr uint64_t kWaitNs = 1000000000ull;
-
 // fp16 pairs per 32-code sub-chunk: every width uses 16 (q=3 merges its two
 // bit planes into 3-bit fields before the mma)
 constexpr int NP = 16;
@@ -20,46 +18,6 @@ constexpr int NP = 16;
 __device__ __forceinline__ uint32_t su32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
-__device__ __forceinline__ uint64_t gtime() {
-  uint64_t t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-__device__ __forceinline__ void bar_init(uint64_t* b, uint32_t c) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(b)), "r"(c) : "memory");
-}
-__device__ __forceinline__ void bar_arrive(uint64_t* b) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(b)) : "memory");
-}
-__device__ __forceinline__ bool bar_try(uint32_t b, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-      " selp.u32 %0, 1, 0, p;\n}\n"
-      : "=r"(ok)
-      : "r"(b), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-// bounded wait; false if it gave up (own limit, or *abort raised elsewhere)
-__device__ __forceinline__ bool bar_wait_a(uint32_t b, uint32_t parity, volatile int* abort) {
-  if (bar_try(b, parity)) return true;
-  const uint64_t t0 = gtime();
-  for (uint32_t it = 1;; ++it) {
-    if (bar_try(b, parity)) return true;
-    if ((it & 255u) == 0) {
-      if (*abort) return false;
-      if (gtime() - t0 > kWaitNs) {
-        *abort = 1;
-        return false;
-      }
-    }
-  }
-}
-__device__ __forceinline__ bool bar_wait(uint64_t* b, uint32_t parity, volatile int* abort) {
-  return bar_wait_a(su32(b), parity, abort);
-}
-
 __device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
                                          uint32_t a3, uint32_t b0, uint32_t b1) {
   asm volatile(
@@ -84,11 +42,6 @@ __device__ __forceinline__ uint4 lds128(uint32_t addr) {
   asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
                : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                : "r"(addr));
-  return v;
-}
-__device__ __forceinline__ float2 lds64f(uint32_t addr) {
-  float2 v;
-  asm volatile("ld.shared.v2.f32 {%0,%1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(addr));
   return v;
 }
 

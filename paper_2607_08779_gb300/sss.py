@@ -409,8 +409,9 @@ def sss_gemm_noalloc_max_scratch_bytes() -> int:
 
 def sss_test_set_stall(mask: int) -> None:
     """Test hook of the bounded waits (TEST_STALL_* bits; 0 restores normal
-    launches): later launches of the named kernels leave one barrier one
-    arrive short, so a wait runs out and the kernel raises FLAG_TIMEOUT."""
+    launches): later GEMM launches leave one barrier one arrive short, so a
+    wait runs out and the kernel raises FLAG_TIMEOUT.  The GEMV kernels have
+    no waits; their bits have no effect."""
     load().sss_test_set_stall(int(mask))
 
 
