@@ -193,11 +193,14 @@ class Workload:
         self.y = [torch.empty((1, n), dtype=torch.float32, device=dev) for _, (n, k) in self.shapes]
         self.Y = [torch.empty((GEMM_M, n), dtype=torch.float32, device=dev)
                   for _, (n, k) in self.shapes]
-        self.ws = {}
-        for mi, (_, (n, k)) in enumerate(self.shapes):
-            need = sss.sss_workspace_bytes(self.fresh_q[4][mi], GEMM_M, sss.OP_GEMM)
-            if need > (self.ws[k].numel() if k in self.ws else -1):
-                self.ws[k] = torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
+        # one workspace per group of matrices sharing X (the GEMM phase runs
+        # each group as one sss_gemm_multi call)
+        idx = {name: i for i, (name, _) in enumerate(self.shapes)}
+        self.ws = []
+        for grp in self.GROUPS:
+            need = sss.sss_gemm_multi_workspace_bytes([self.fresh_q[4][idx[nm]] for nm in grp],
+                                                      GEMM_M)
+            self.ws.append(torch.empty(max(need, 16), dtype=torch.uint8, device=dev))
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
         torch.cuda.synchronize()
 
@@ -218,8 +221,9 @@ class Workload:
         self.quant_bytes = sum(4 * n * k + n * k * q // 8 + 2 * n * (k // GROUP)
                                for q in QS for _, (n, k) in self.shapes)
         self.gemm_flops = 2 * GEMM_M * sum(n * k for _, (n, k) in self.shapes)
+        # quantize, GEMV, and per GEMM group the X conversion and the GEMM
         self.launches_per_step = (len(QS) * len(self.shapes) + self.gemv_launches
-                                  + 2 * len(self.shapes))
+                                  + 2 * len(self.GROUPS))
 
     # -- phases (each captured once as a CUDA graph) --
     def quantize_phase(self, f: int):
@@ -247,10 +251,16 @@ class Workload:
                     sss.sss_gemv_multi([self.stack[q][layer][mi] for mi in mis], self.x[k][0],
                                        ys=[self.y[mi][0] for mi in mis], flags=flags)
 
+    # prefill of GEMM_M tokens through the layer's matrices, the ones that
+    # share X in one launch: {q, k, v}, o, {gate, up}, down
     def gemm_phase(self):
-        for mi, (_, (n, k)) in enumerate(self.shapes):
-            self.sss.sss_gemm(self.fresh_q[4][mi], self.X[k], y=self.Y[mi], workspace=self.ws[k],
-                              dev_status=self.status)
+        idx = {name: i for i, (name, _) in enumerate(self.shapes)}
+        for gi, grp in enumerate(self.GROUPS):
+            mis = [idx[nm] for nm in grp]
+            k = self.shapes[mis[0]][1][1]
+            self.sss.sss_gemm_multi([self.fresh_q[4][mi] for mi in mis], self.X[k],
+                                    ys=[self.Y[mi] for mi in mis], workspace=self.ws[gi],
+                                    dev_status=self.status)
 
     def capture(self):
         torch = self.torch
@@ -714,7 +724,8 @@ def run_micro(args):
     ys = [torch.empty((rows_x, n), dtype=torch.float32, device="cuda") for n, _ in shapes]
     ws = None
     if args.micro == "gemm":
-        need = max(sss.sss_workspace_bytes(qt, args.m, sss.OP_GEMM) for qt in copies[0])
+        need = (sss.sss_gemm_multi_workspace_bytes(copies[0], args.m) if args.fuse else
+                max(sss.sss_workspace_bytes(qt, args.m, sss.OP_GEMM) for qt in copies[0]))
         ws = torch.empty(max(need, 16), dtype=torch.uint8, device="cuda")
 
     def op(c):
@@ -724,6 +735,8 @@ def run_micro(args):
         elif args.micro == "gemv_single":
             for qt, y in zip(mats, ys):
                 sss.sss_gemv(qt, x, y=y)
+        elif args.micro == "gemm" and args.fuse:
+            sss.sss_gemm_multi(mats, x, ys=ys, workspace=ws)
         elif args.micro == "gemm":
             for qt, y in zip(mats, ys):
                 sss.sss_gemm(qt, x, y=y, workspace=ws)
@@ -761,7 +774,8 @@ def run_micro(args):
         nbytes += 2 * k * rows_x
     flops = 2 * rows_x * sum(n * kk for n, kk in shapes)
     print(json.dumps({"micro": args.micro, "matrices": names, "q": q, "group": g, "rows_x": rows_x,
-                      "grid": args.grid, "us_per_call": round(us, 3),
+                      "grid": args.grid, "fused": bool(getattr(args, "fuse", False)),
+                      "us_per_call": round(us, 3),
                       "gbs": round(nbytes / us / 1e3, 1), "tflops": round(flops / us / 1e6, 2),
                       "iters": args.iters, "rotate": args.rotate}), flush=True)
 
@@ -991,6 +1005,8 @@ def main():
     ap.add_argument("--iters", type=int, default=50)
     ap.add_argument("--rotate", type=int, default=8)
     ap.add_argument("--flags", type=int, default=0)
+    ap.add_argument("--fuse", action="store_true",
+                    help="micro gemm: the matrices in one sss_gemm_multi call")
     ap.add_argument("--rows", type=int, default=0, help="micro: override every matrix's rows")
     ap.add_argument("--sweep", choices=["qwen3_quantize", "grids", "margins"],
                     help="measurement sweeps: whole-model quantization of Qwen3-32B shapes, "

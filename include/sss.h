@@ -236,6 +236,34 @@ sss_status_t sss_gemm(const sss_qtensor_t* qt, const uint16_t* x_bf16,
                       uint32_t* dev_status, void* stream);
 
 /*
+ * sss_gemm_multi -- sss_gemm for several packed matrices that share one
+ * activation matrix (e.g. the q/k/v or gate/up projections of a layer) in
+ * one launch: Y_j[m][r] = sum_k w^_j[r][k] * X[m][k] (same arithmetic as
+ * sss_gemm, Appendix B.3).  X is converted to fp16 once, and the output
+ * tiles of all the matrices share one grid, so small matrices (k/v) fill
+ * the SMs together with the others instead of splitting K.
+ *   qts   [in]  count pointers to packed tensors with equal k, q, group and
+ *               grid; each n % 4 == 0; codes 16-byte aligned.  Tensors with
+ *               n == 0 are skipped.
+ *   ys    [out] count device fp32 pointers, Y_j [m][n_j], 16-byte aligned.
+ *   count [in]  1..4.
+ *   x_bf16, m, workspace, ws_bytes, dev_status, stream: as sss_gemm, with
+ *               the workspace sized by sss_gemm_multi_workspace_bytes (the
+ *               fp16 copy of X, m*k*2 bytes, is enough to run unsplit).
+ * Errors: SSS_E_ARG (count, mismatched tensors), SSS_E_ALIGN,
+ * SSS_E_UNSUPPORTED, SSS_E_WORKSPACE, SSS_E_CUDA.
+ */
+sss_status_t sss_gemm_multi(const sss_qtensor_t* const* qts, float* const* ys,
+                            int32_t count, const uint16_t* x_bf16, int64_t m,
+                            void* workspace, size_t ws_bytes,
+                            uint32_t* dev_status, void* stream);
+
+/* Workspace bytes that let sss_gemm_multi take its preferred plan (0 for
+ * invalid arguments or an empty call). */
+size_t sss_gemm_multi_workspace_bytes(const sss_qtensor_t* const* qts,
+                                      int32_t count, int64_t m);
+
+/*
  * sss_gemm_q8 -- sss_gemm on Q8_0 activations: each token's X is quantized
  * per block of 32 (sss_quantize_act_q8) and the GEMM multiplies the packed
  * weights with fl16(fl16(d) * q), the fp16 operand of the tensor cores (one

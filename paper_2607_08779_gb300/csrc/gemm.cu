@@ -41,6 +41,8 @@
 // the tensor memory is still released.
 #include <cuda.h>
 
+#include <string.h>
+
 #include <algorithm>
 #include <mutex>
 
@@ -266,21 +268,40 @@ __device__ __forceinline__ void load_sub32(const uint8_t* __restrict__ row, int6
   }
 }
 
-struct GemmArgs {
+// One weight matrix of a call (several share X, e.g. a fused q/k/v
+// projection): its row tiles are tiles tile0 .. tile0 + ceil(n / 128) - 1 of
+// the grid's x dimension.
+struct GemmJob {
   const uint8_t* codes;
   const uint16_t* scales;
   const uint16_t* mins;
-  float* y;
+  float* y;  // [m][n]
+  int64_t n;
+  int64_t tile0;
+};
+struct GemmArgs {
+  GemmJob job[kMaxGemmJobs];
+  int njobs;
   uint32_t* status;
-  int64_t m, n, k;
+  int64_t m, k;
   int G;
   int stall;  // test hook: the first stage's weight tile is never announced
   // split K: CTA z of nsplit takes k-blocks [z * chunk, ...) and leaves its
-  // fp32 tile in part + z * m * n; the last of a tile's splits to finish
+  // fp32 tile in part + z * m * np (row tile t at rows 128 t .. 128 t + 127
+  // of np = 128 x all row tiles); the last of a tile's splits to finish
   // (counted in cnt, zero on entry) sums them in split order into y
   int nsplit;
+  int64_t np;
   float* part;
   int* cnt;
+};
+
+// The activation tile map, and per matrix its code and scale tile maps
+// (used with TW).
+struct GemmMaps {
+  CUtensorMap x;
+  CUtensorMap c[kMaxGemmJobs];
+  CUtensorMap s[kMaxGemmJobs];
 };
 
 // Shared memory: STAGES activation tiles (1024-aligned for the 128-byte
@@ -310,8 +331,7 @@ constexpr int tmem_cols_of() { return SETS == 1 ? 256 : 512; }
 // memory a few k-blocks ahead.
 template <int Q, bool ASYM, int BN, int STAGES, bool TW, int SETS>
 __global__ void __launch_bounds__(threads_of<SETS>(), SETS == 1 ? 2 : 1)
-    gemm_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap cmap,
-                const __grid_constant__ CUtensorMap smap, const GemmArgs a) {
+    gemm_kernel(const __grid_constant__ GemmMaps maps, const __grid_constant__ GemmArgs a) {
   using S = Smem<BN, STAGES, Q, TW>;
   constexpr int kTmemCols = tmem_cols_of<SETS>();
   static_assert(BN + 32 * STAGES <= kTmemCols, "tensor memory holds the accumulator and A stages");
@@ -328,7 +348,13 @@ __global__ void __launch_bounds__(threads_of<SETS>(), SETS == 1 ? 2 : 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int64_t n0 = static_cast<int64_t>(blockIdx.x) * kBM;
+  // this CTA's matrix jb, its rows n0 .. n0 + 127 in that matrix, and the
+  // same rows g0 .. g0 + 127 of the partial tiles
+  int jb = 0;
+  while (jb + 1 < a.njobs && static_cast<int64_t>(blockIdx.x) >= a.job[jb + 1].tile0) ++jb;
+  const GemmJob& job = a.job[jb];
+  const int64_t n0 = (static_cast<int64_t>(blockIdx.x) - job.tile0) * kBM;
+  const int64_t g0 = static_cast<int64_t>(blockIdx.x) * kBM;
   const int64_t m0 = static_cast<int64_t>(blockIdx.y) * BN;
   // this split's k-blocks: global k-block kb_base + kb for kb = 0 .. nkb - 1
   const int nkb_all = static_cast<int>(a.k / kBK);
@@ -373,13 +399,13 @@ __global__ void __launch_bounds__(threads_of<SETS>(), SETS == 1 ? 2 : 1)
         if (!mbar_wait(&empty[s], ph ^ 1u, abort)) break;
         unsigned char* sb = smem + s * S::STAGE;
         mbar_arrive_expect_tx(&full_b[s], S::B_BYTES + S::C_BYTES + S::S_BYTES);
-        tma_load_2d(&xmap, &full_b[s], sb, (kb_base + kb) * kBK, static_cast<int>(m0));
+        tma_load_2d(&maps.x, &full_b[s], sb, (kb_base + kb) * kBK, static_cast<int>(m0));
         if constexpr (TW) {
           // the k-block's codes (8q bytes of each row, x a multiple of 16) and
           // the 8-scale window holding its groups (x rounded down to 8)
-          tma_load_2d(&cmap, &full_b[s], smem + S::C_OFF + s * S::C_BYTES,
+          tma_load_2d(&maps.c[jb], &full_b[s], smem + S::C_OFF + s * S::C_BYTES,
                       (kb_base + kb) * 8 * Q, static_cast<int>(n0));
-          tma_load_2d(&smap, &full_b[s], smem + S::S_OFF + s * S::S_BYTES,
+          tma_load_2d(&maps.s[jb], &full_b[s], smem + S::S_OFF + s * S::S_BYTES,
                       ((kb_base + kb) * kBK / a.G) & ~7, static_cast<int>(n0));
         }
         issued = kb + 1;
@@ -422,10 +448,6 @@ __global__ void __launch_bounds__(threads_of<SETS>(), SETS == 1 ? 2 : 1)
     const int row_i = 32 * (warp & 3) + lane;
     const int hf = ((warp - 2) >> 2) & 1;
     const int set = (warp - 2) >> 3;
-    const int64_t r = n0 + row_i;
-    const bool rok = r < a.n;
-    const int64_t nG = a.k / a.G;
-    const uint8_t* rowp = a.codes + (rok ? r : 0) * (a.k * Q / 8);
     bool big = false;  // a group whose s*c may leave the fp16 range
     bool ok = true;
     // fp16 s*c (ASYM: s*u + m) of the thread's 32 codes w into stage s's A
@@ -501,9 +523,9 @@ __global__ void __launch_bounds__(threads_of<SETS>(), SETS == 1 ? 2 : 1)
       }
     } else {
       const int64_t r = n0 + row_i;
-      const bool rok = r < a.n;
+      const bool rok = r < job.n;
       const int64_t nG = a.k / a.G;
-      const uint8_t* rowp = a.codes + (rok ? r : 0) * (a.k * Q / 8);
+      const uint8_t* rowp = job.codes + (rok ? r : 0) * (a.k * Q / 8);
       // codes and scale (and min) of this thread's half of one k-block
       struct KBlock {
         uint32_t w[4];
@@ -515,8 +537,8 @@ __global__ void __launch_bounds__(threads_of<SETS>(), SETS == 1 ? 2 : 1)
         const int64_t grp = kc / a.G;
         const int sc = static_cast<int>((kc % a.G) / 32);
         load_sub32<Q>(rowp, grp, sc, a.G, rok, d.w);
-        d.s = rok ? __ldcs(a.scales + r * nG + grp) : static_cast<uint16_t>(0);
-        if constexpr (ASYM) d.m = rok ? __ldcs(a.mins + r * nG + grp) : static_cast<uint16_t>(0);
+        d.s = rok ? __ldcs(job.scales + r * nG + grp) : static_cast<uint16_t>(0);
+        if constexpr (ASYM) d.m = rok ? __ldcs(job.mins + r * nG + grp) : static_cast<uint16_t>(0);
       };
       // the global loads run kPrefetch of this thread's k-blocks ahead of use
       constexpr int kPrefetch = 4;
@@ -560,12 +582,15 @@ __global__ void __launch_bounds__(threads_of<SETS>(), SETS == 1 ? 2 : 1)
         uint32_t v[32];
         tmem_ld32(tmem + (static_cast<uint32_t>(sub * 32) << 16) + c0, v);
         // one split: y; several: this split's partial tile
-        float* dst = a.nsplit > 1 ? a.part + static_cast<int64_t>(blockIdx.z) * a.m * a.n : a.y;
-        if (rr < a.n) {
+        const bool split = a.nsplit > 1;
+        float* dst = split ? a.part + static_cast<int64_t>(blockIdx.z) * a.m * a.np + g0 + row_local
+                           : job.y + rr;
+        const int64_t ld = split ? a.np : job.n;
+        if (rr < job.n) {
 #pragma unroll
           for (int c = 0; c < 32; ++c) {
             const int64_t mm = m0 + c0 + c;
-            if (mm < a.m) dst[mm * a.n + rr] = __uint_as_float(v[c]);
+            if (mm < a.m) dst[mm * ld] = __uint_as_float(v[c]);
           }
         }
       }
@@ -591,7 +616,7 @@ __global__ void __launch_bounds__(threads_of<SETS>(), SETS == 1 ? 2 : 1)
       // split's eight loads are in flight together
       constexpr int kV = kBM / 4;  // float4 per token of the tile
       constexpr int kE = 8;
-      const int64_t mn = a.m * a.n;
+      const int64_t mn = a.m * a.np;
       for (int e0 = threadIdx.x; e0 < kV * BN; e0 += kE * blockDim.x) {
         float4 acc[kE];
         int64_t off[kE];
@@ -600,8 +625,8 @@ __global__ void __launch_bounds__(threads_of<SETS>(), SETS == 1 ? 2 : 1)
         for (int j = 0; j < kE; ++j) {
           const int e = e0 + j * blockDim.x;
           const int64_t mm = m0 + e / kV, rr = n0 + 4 * (e % kV);
-          in[j] = e < kV * BN && mm < a.m && rr < a.n;
-          off[j] = in[j] ? mm * a.n + rr : 0;
+          in[j] = e < kV * BN && mm < a.m && rr < job.n;
+          off[j] = in[j] ? mm * a.np + g0 + 4 * (e % kV) : 0;
           acc[j] = in[j] ? __ldcg(reinterpret_cast<const float4*>(a.part + off[j]))
                          : make_float4(0.f, 0.f, 0.f, 0.f);
         }
@@ -617,8 +642,11 @@ __global__ void __launch_bounds__(threads_of<SETS>(), SETS == 1 ? 2 : 1)
           }
         }
 #pragma unroll
-        for (int j = 0; j < kE; ++j)
-          if (in[j]) *reinterpret_cast<float4*>(a.y + off[j]) = acc[j];
+        for (int j = 0; j < kE; ++j) {
+          const int e = e0 + j * blockDim.x;
+          if (in[j])
+            *reinterpret_cast<float4*>(job.y + (m0 + e / kV) * job.n + n0 + 4 * (e % kV)) = acc[j];
+        }
       }
       if (threadIdx.x == 0) *cnt = 0;
     }
@@ -677,22 +705,22 @@ struct GemmPlan {
   int bn, sets, nsplit;
 };
 
-// Workspace layout: fp16 X, then (split K) the partial tiles, then the
+// Workspace layout: fp16 X, then (split K) the partial tiles (rows padded to
+// whole row tiles, rt of them over all the call's matrices), then the
 // per-tile counters.
 size_t round256(size_t b) { return (b + 255) / 256 * 256; }
-size_t split_bytes(const sss_qtensor_t& t, int64_t m, const GemmPlan& p) {
+size_t split_bytes(int64_t rt, int64_t m, const GemmPlan& p) {
   if (p.nsplit <= 1) return 0;
-  const size_t tiles = static_cast<size_t>((t.n + kBM - 1) / kBM) * ((m + p.bn - 1) / p.bn);
-  return round256(static_cast<size_t>(p.nsplit) * m * t.n * 4) + round256(tiles * 4);
+  const size_t tiles = static_cast<size_t>(rt) * ((m + p.bn - 1) / p.bn);
+  return round256(static_cast<size_t>(p.nsplit) * m * rt * kBM * 4) + round256(tiles * 4);
 }
 
 // Largest K split (>= 2 to count) that fills the idle SMs with `tiles`
 // tiles, keeps every split non-empty and at least `min_kb` k-blocks long,
 // and whose partial tiles fit in the workspace (ws bytes); 1 if none.
-int split_for(const sss_qtensor_t& t, int64_t m, size_t ws, int bn, int64_t tiles,
-              int64_t min_kb) {
+int split_for(int64_t k, int64_t rt, int64_t m, size_t ws, int bn, int64_t tiles, int64_t min_kb) {
   const int64_t sms = device_sm_count();
-  const int64_t nkb = t.k / kBK;
+  const int64_t nkb = k / kBK;
   int split = static_cast<int>(std::min<int64_t>(sms / std::max<int64_t>(tiles, 1), nkb / min_kb));
   if (split >= 2) {  // every split non-empty: as many as chunks of ceil(nkb / split)
     const int64_t chunk = (nkb + split - 1) / split;
@@ -700,7 +728,7 @@ int split_for(const sss_qtensor_t& t, int64_t m, size_t ws, int bn, int64_t tile
   }
   for (; split >= 2; --split) {
     const GemmPlan p{bn, 2, split};
-    if (x16_bytes(m, t.k) <= ws && x16_bytes(m, t.k) + split_bytes(t, m, p) <= ws) return split;
+    if (x16_bytes(m, k) <= ws && x16_bytes(m, k) + split_bytes(rt, m, p) <= ws) return split;
   }
   return 1;
 }
@@ -713,81 +741,98 @@ int split_for(const sss_qtensor_t& t, int64_t m, size_t ws, int bn, int64_t tile
 // SMs idle.  The tile's last split sums all partials alone, so a split pays
 // only with enough k-blocks behind it.  (Two half-size CTAs per SM, one
 // dequantising set each, measured slower than one full CTA: their rings are
-// half as deep.)
-GemmPlan plan_gemm(const sss_qtensor_t& t, int64_t m, size_t ws) {
+// half as deep.)  rt: the row tiles of all the call's matrices.
+GemmPlan plan_gemm(int64_t rt, int64_t k, int64_t m, size_t ws) {
   const int64_t sms = device_sm_count();
-  const int64_t rt = (t.n + kBM - 1) / kBM;
   if (m > 128) {
     const int64_t tiles = rt * ((m + 255) / 256);
     if (tiles >= sms) return {256, 2, 1};
-    const int split = split_for(t, m, ws, 256, tiles, 64);
+    const int split = split_for(k, rt, m, ws, 256, tiles, 64);
     if (split >= 2) return {256, 2, split};
   }
   const int64_t tiles = rt * ((m + 127) / 128);
   if (tiles >= sms) return {128, 2, 1};
-  return {128, 2, split_for(t, m, ws, 128, tiles, 8)};
+  return {128, 2, split_for(k, rt, m, ws, 128, tiles, 8)};
+}
+
+int64_t row_tiles(const sss_qtensor_t* const* ts, int count) {
+  int64_t rt = 0;
+  for (int j = 0; j < count; ++j) rt += (ts[j]->n + kBM - 1) / kBM;
+  return rt;
 }
 
 template <int Q, bool ASYM, int BN, bool TW, int SETS>
-cudaError_t run_gemm(const sss_qtensor_t& t, const __half* x16, int64_t m, float* y,
-                     uint32_t* status, cudaStream_t stream, int nsplit, unsigned char* ws_split) {
+cudaError_t run_gemm(const sss_qtensor_t* const* ts, float* const* ys, int count,
+                     const __half* x16, int64_t m, uint32_t* status, cudaStream_t stream,
+                     int nsplit, unsigned char* ws_split) {
   constexpr int STAGES = (BN == 256) ? (TW ? 5 : 6) : 8;
   using S = Smem<BN, STAGES, Q, TW>;
+  const sss_qtensor_t& t0 = *ts[0];  // k, q, group and grid are those of every matrix
   EncodeTiledFn enc = tensor_map_encoder();
   if (enc == nullptr) return cudaErrorNotSupported;
-  CUtensorMap map;
-  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(t.k), static_cast<cuuint64_t>(m)};
-  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(t.k) * 2};
+  GemmMaps maps;
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(t0.k), static_cast<cuuint64_t>(m)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(t0.k) * 2};
   const cuuint32_t box[2] = {kBK, BN};
   const cuuint32_t estr[2] = {1, 1};
-  CUresult cr = enc(&map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<__half*>(x16), dims,
+  CUresult cr = enc(&maps.x, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<__half*>(x16), dims,
                     strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                     CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
-  CUtensorMap cmap = map, smap = map;
-  if constexpr (TW) {
-    // packed codes [n][k q / 8] bytes: one k-block is 8q bytes of 128 rows;
-    // scales [n][k / G] fp16: a window of 8 (16 bytes) of 128 rows; rows
-    // past n read as zero
-    const cuuint64_t cd[2] = {static_cast<cuuint64_t>(t.k * Q / 8), static_cast<cuuint64_t>(t.n)};
-    const cuuint64_t cs[1] = {static_cast<cuuint64_t>(t.k * Q / 8)};
-    const cuuint32_t cb[2] = {static_cast<cuuint32_t>(8 * Q), kBM};
-    cr = enc(&cmap, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, t.codes, cd, cs, cb, estr,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
-    const int64_t ng = t.k / t.group;
-    const cuuint64_t sd[2] = {static_cast<cuuint64_t>(ng), static_cast<cuuint64_t>(t.n)};
-    const cuuint64_t ss[1] = {static_cast<cuuint64_t>(ng * 2)};
-    const cuuint32_t sbx[2] = {8, kBM};
-    cr = enc(&smap, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, t.scales, sd, ss, sbx, estr,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
+  GemmArgs a;
+  memset(&a, 0, sizeof a);
+  int64_t tile0 = 0;
+  for (int j = 0; j < count; ++j) {
+    const sss_qtensor_t& t = *ts[j];
+    maps.c[j] = maps.x;  // placeholders unless TW
+    maps.s[j] = maps.x;
+    if constexpr (TW) {
+      // packed codes [n][k q / 8] bytes: one k-block is 8q bytes of 128 rows;
+      // scales [n][k / G] fp16: a window of 8 (16 bytes) of 128 rows; rows
+      // past n read as zero
+      const cuuint64_t cd[2] = {static_cast<cuuint64_t>(t.k * Q / 8), static_cast<cuuint64_t>(t.n)};
+      const cuuint64_t cs[1] = {static_cast<cuuint64_t>(t.k * Q / 8)};
+      const cuuint32_t cb[2] = {static_cast<cuuint32_t>(8 * Q), kBM};
+      cr = enc(&maps.c[j], CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, t.codes, cd, cs, cb, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+      if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
+      const int64_t ng = t.k / t.group;
+      const cuuint64_t sd[2] = {static_cast<cuuint64_t>(ng), static_cast<cuuint64_t>(t.n)};
+      const cuuint64_t ss[1] = {static_cast<cuuint64_t>(ng * 2)};
+      const cuuint32_t sbx[2] = {8, kBM};
+      cr = enc(&maps.s[j], CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, t.scales, sd, ss, sbx, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+      if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    }
+    a.job[j].codes = t.codes;
+    a.job[j].scales = t.scales;
+    a.job[j].mins = t.mins;
+    a.job[j].y = ys[j];
+    a.job[j].n = t.n;
+    a.job[j].tile0 = tile0;
+    tile0 += (t.n + kBM - 1) / kBM;
   }
   auto kern = gemm_kernel<Q, ASYM, BN, STAGES, TW, SETS>;
   cudaError_t e = ensure_smem(kern, S::TOTAL);
   if (e != cudaSuccess) return e;
-  GemmArgs a;
-  a.codes = t.codes;
-  a.scales = t.scales;
-  a.mins = t.mins;
-  a.y = y;
+  a.njobs = count;
   a.status = status;
   a.m = m;
-  a.n = t.n;
-  a.k = t.k;
-  a.G = t.group;
+  a.k = t0.k;
+  a.G = t0.group;
   a.stall = (test_stall_mask() & SSS_TEST_STALL_GEMM) ? 1 : 0;
   a.nsplit = nsplit;
+  a.np = tile0 * kBM;
   a.part = nullptr;
   a.cnt = nullptr;
-  const unsigned gx = static_cast<unsigned>((t.n + kBM - 1) / kBM);
+  const unsigned gx = static_cast<unsigned>(tile0);
   const unsigned gy = static_cast<unsigned>((m + BN - 1) / BN);
   if (nsplit > 1) {
     a.part = reinterpret_cast<float*>(ws_split);
-    a.cnt = reinterpret_cast<int*>(ws_split + round256(static_cast<size_t>(nsplit) * m * t.n * 4));
+    a.cnt = reinterpret_cast<int*>(ws_split + round256(static_cast<size_t>(nsplit) * m * a.np * 4));
     e = cudaMemsetAsync(a.cnt, 0, sizeof(int) * gx * gy, stream);
     if (e != cudaSuccess) return e;
   }
@@ -801,61 +846,79 @@ cudaError_t run_gemm(const sss_qtensor_t& t, const __half* x16, int64_t m, float
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kern, map, cmap, smap, a);
+  return cudaLaunchKernelEx(&cfg, kern, maps, a);
 }
 
+struct GemmCall {
+  const sss_qtensor_t* const* ts;
+  float* const* ys;
+  int count;
+  const __half* x16;
+  int64_t m;
+  uint32_t* status;
+  cudaStream_t stream;
+  GemmPlan plan;
+  unsigned char* ws_split;
+};
+
 template <int Q, bool ASYM, bool TW>
-cudaError_t gemm_tw(const sss_qtensor_t& t, const __half* x16, int64_t m, float* y,
-                    uint32_t* status, cudaStream_t stream, const GemmPlan& p,
-                    unsigned char* ws_split) {
-  if (p.bn == 256)
-    return run_gemm<Q, ASYM, 256, TW, 2>(t, x16, m, y, status, stream, p.nsplit, ws_split);
-  return run_gemm<Q, ASYM, 128, TW, 2>(t, x16, m, y, status, stream, p.nsplit, ws_split);
+cudaError_t gemm_tw(const GemmCall& c) {
+  if (c.plan.bn == 256)
+    return run_gemm<Q, ASYM, 256, TW, 2>(c.ts, c.ys, c.count, c.x16, c.m, c.status, c.stream,
+                                         c.plan.nsplit, c.ws_split);
+  return run_gemm<Q, ASYM, 128, TW, 2>(c.ts, c.ys, c.count, c.x16, c.m, c.status, c.stream,
+                                       c.plan.nsplit, c.ws_split);
 }
 
 template <int Q, bool ASYM>
-cudaError_t gemm_bn(const sss_qtensor_t& t, const __half* x16, int64_t m, float* y,
-                    uint32_t* status, cudaStream_t stream, const GemmPlan& p,
-                    unsigned char* ws_split) {
+cudaError_t gemm_bn(const GemmCall& c) {
   if constexpr (!ASYM && Q != 3) {
-    // the code and scale tiles by TMA: 16-byte aligned scale rows
-    const bool tw = (reinterpret_cast<uintptr_t>(t.scales) % 16) == 0 &&
-                    ((t.k / t.group) * 2) % 16 == 0;
-    if (tw) return gemm_tw<Q, ASYM, true>(t, x16, m, y, status, stream, p, ws_split);
+    // the code and scale tiles by TMA: 16-byte aligned scale rows in every
+    // matrix
+    bool tw = ((c.ts[0]->k / c.ts[0]->group) * 2) % 16 == 0;
+    for (int j = 0; j < c.count; ++j)
+      tw = tw && (reinterpret_cast<uintptr_t>(c.ts[j]->scales) % 16) == 0;
+    if (tw) return gemm_tw<Q, ASYM, true>(c);
   }
-  return gemm_tw<Q, ASYM, false>(t, x16, m, y, status, stream, p, ws_split);
+  return gemm_tw<Q, ASYM, false>(c);
 }
 
 template <int Q>
-cudaError_t gemm_grid(const sss_qtensor_t& t, const __half* x16, int64_t m, float* y,
-                      uint32_t* status, cudaStream_t stream, const GemmPlan& p,
-                      unsigned char* ws_split) {
-  if (t.grid == SSS_GRID_ASYM) return gemm_bn<Q, true>(t, x16, m, y, status, stream, p, ws_split);
-  return gemm_bn<Q, false>(t, x16, m, y, status, stream, p, ws_split);
+cudaError_t gemm_grid(const GemmCall& c) {
+  if (c.ts[0]->grid == SSS_GRID_ASYM) return gemm_bn<Q, true>(c);
+  return gemm_bn<Q, false>(c);
 }
 
 }  // namespace
 
 // the workspace that lets the call take its preferred plan (with split K
 // where it helps); x16_bytes alone is enough to run it unsplit
-size_t gemm_workspace_bytes(const sss_qtensor_t& t, int64_t m) {
-  const size_t x = x16_bytes(m, t.k);
+size_t gemm_multi_workspace_bytes(const sss_qtensor_t* const* ts, int count, int64_t m) {
+  const size_t x = x16_bytes(m, ts[0]->k);
   if (x == SIZE_MAX) return SIZE_MAX;
-  return x + split_bytes(t, m, plan_gemm(t, m, SIZE_MAX));
+  const int64_t rt = row_tiles(ts, count);
+  return x + split_bytes(rt, m, plan_gemm(rt, ts[0]->k, m, SIZE_MAX));
+}
+size_t gemm_workspace_bytes(const sss_qtensor_t& t, int64_t m) {
+  const sss_qtensor_t* one[1] = {&t};
+  return gemm_multi_workspace_bytes(one, 1, m);
 }
 size_t gemm_workspace_min_bytes(const sss_qtensor_t& t, int64_t m) { return x16_bytes(m, t.k); }
 
-cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m, float* y,
-                        void* workspace, size_t ws_bytes, uint32_t* status, cudaStream_t stream,
-                        bool act_q8) {
+cudaError_t launch_gemm_multi(const sss_qtensor_t* const* ts, float* const* ys, int count,
+                              const uint16_t* x, int64_t m, void* workspace, size_t ws_bytes,
+                              uint32_t* status, cudaStream_t stream, bool act_q8) {
+  if (count < 1 || count > kMaxGemmJobs) return cudaErrorInvalidValue;
+  const int64_t k = ts[0]->k;
   __half* x16 = static_cast<__half*>(workspace);
-  const GemmPlan plan = plan_gemm(t, m, ws_bytes);
-  unsigned char* ws_split = static_cast<unsigned char*>(workspace) + x16_bytes(m, t.k);
+  const int64_t rt = row_tiles(ts, count);
+  const GemmPlan plan = plan_gemm(rt, k, m, ws_bytes);
+  unsigned char* ws_split = static_cast<unsigned char*>(workspace) + x16_bytes(m, k);
   cudaError_t e;
   if (act_q8) {
-    e = launch_act_q8_f16(x, m, t.k, x16, status, stream);
+    e = launch_act_q8_f16(x, m, k, x16, status, stream);
   } else {
-    const int64_t nvec = m * t.k / 8;
+    const int64_t nvec = m * k / 8;
     const int grid = static_cast<int>(std::min<int64_t>((nvec + 255) / 256,
                                                         static_cast<int64_t>(device_sm_count()) * 8));
     cudaLaunchConfig_t cfg = {};
@@ -870,12 +933,21 @@ cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m, fl
     e = cudaLaunchKernelEx(&cfg, bf16_to_f16_kernel, x, x16, nvec);
   }
   if (e != cudaSuccess) return e;
-  switch (t.q) {
-    case 2: return gemm_grid<2>(t, x16, m, y, status, stream, plan, ws_split);
-    case 3: return gemm_grid<3>(t, x16, m, y, status, stream, plan, ws_split);
-    case 4: return gemm_grid<4>(t, x16, m, y, status, stream, plan, ws_split);
+  const GemmCall c{ts, ys, count, x16, m, status, stream, plan, ws_split};
+  switch (ts[0]->q) {
+    case 2: return gemm_grid<2>(c);
+    case 3: return gemm_grid<3>(c);
+    case 4: return gemm_grid<4>(c);
   }
   return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m, float* y,
+                        void* workspace, size_t ws_bytes, uint32_t* status, cudaStream_t stream,
+                        bool act_q8) {
+  const sss_qtensor_t* one[1] = {&t};
+  float* ys[1] = {y};
+  return launch_gemm_multi(one, ys, 1, x, m, workspace, ws_bytes, status, stream, act_q8);
 }
 
 }  // namespace sss

@@ -282,6 +282,75 @@ sss_status_t sss_gemm(const sss_qtensor_t* qt, const uint16_t* x_bf16, int64_t m
                      false);
 }
 
+namespace {
+// the matrices of one sss_gemm_multi call: valid, alike in k, q, group and
+// grid, each with n % 4 == 0 and aligned buffers; the ones with rows kept
+sss_status_t gemm_multi_jobs(const sss_qtensor_t* const* qts, float* const* ys, int32_t count,
+                             const sss_qtensor_t** keep, float** keep_y, int* kept) {
+  if (qts == nullptr || count < 1 || count > kMaxGemmJobs) return SSS_E_ARG;
+  *kept = 0;
+  for (int j = 0; j < count; ++j) {
+    sss_status_t st = check_tensor(qts[j]);
+    if (st != SSS_OK) return st;
+    const sss_qtensor_t& t = *qts[j];
+    const sss_qtensor_t& t0 = *qts[0];
+    if (t.k != t0.k || t.q != t0.q || t.group != t0.group || t.grid != t0.grid) return SSS_E_ARG;
+    if (t.n == 0) continue;
+    if (keep_y != nullptr) {
+      if (ys == nullptr || ys[j] == nullptr) return SSS_E_ARG;
+      if (t.k > 0 && t.n % 4 != 0) return SSS_E_UNSUPPORTED;
+      if (!aligned(ys[j], 16)) return SSS_E_ALIGN;
+      if (t.k > 0 && (!aligned(t.codes, 16) || !aligned(t.scales, 2) ||
+                      (t.mins && !aligned(t.mins, 2))))
+        return SSS_E_ALIGN;
+      keep_y[*kept] = ys[j];
+    }
+    keep[(*kept)++] = qts[j];
+  }
+  return SSS_OK;
+}
+}  // namespace
+
+size_t sss_gemm_multi_workspace_bytes(const sss_qtensor_t* const* qts, int32_t count,
+                                      int64_t m) {
+  const sss_qtensor_t* keep[kMaxGemmJobs];
+  int kept = 0;
+  if (m < 0 || gemm_multi_jobs(qts, nullptr, count, keep, nullptr, &kept) != SSS_OK) return 0;
+  if (kept == 0 || m == 0) return 0;
+  return gemm_multi_workspace_bytes(keep, kept, m);
+}
+
+sss_status_t sss_gemm_multi(const sss_qtensor_t* const* qts, float* const* ys, int32_t count,
+                            const uint16_t* x_bf16, int64_t m, void* workspace, size_t ws_bytes,
+                            uint32_t* dev_status, void* stream) {
+  const sss_qtensor_t* keep[kMaxGemmJobs];
+  float* keep_y[kMaxGemmJobs];
+  int kept = 0;
+  sss_status_t st = gemm_multi_jobs(qts, ys, count, keep, keep_y, &kept);
+  if (st != SSS_OK) return st;
+  if (m < 0 || m > kMaxTokens) return SSS_E_ARG;
+  if (m == 0 || kept == 0) return SSS_OK;
+  if (x_bf16 == nullptr) return SSS_E_ARG;
+  const int64_t k = keep[0]->k;
+  if (k % 64 != 0) return SSS_E_UNSUPPORTED;
+  if (!aligned(x_bf16, 16)) return SSS_E_ALIGN;
+  if (dev_status && !aligned(dev_status, 4)) return SSS_E_ALIGN;
+  const size_t need = gemm_workspace_min_bytes(*keep[0], m);
+  if (need > 0 && (workspace == nullptr || ws_bytes < need)) return SSS_E_WORKSPACE;
+  if (workspace != nullptr && !aligned(workspace, 16)) return SSS_E_ALIGN;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (k == 0) {
+    for (int j = 0; j < kept; ++j) {
+      const cudaError_t e =
+          cudaMemsetAsync(keep_y[j], 0, sizeof(float) * static_cast<size_t>(m) * keep[j]->n, s);
+      if (e != cudaSuccess) return finish("sss_gemm_multi", e);
+    }
+    return SSS_OK;
+  }
+  return finish("sss_gemm_multi", launch_gemm_multi(keep, keep_y, kept, x_bf16, m, workspace,
+                                                    ws_bytes, dev_status, s, false));
+}
+
 sss_status_t sss_gemm_q8(const sss_qtensor_t* qt, const uint16_t* x_bf16, int64_t m,
                          float* y, void* workspace, size_t ws_bytes,
                          uint32_t* dev_status, void* stream) {

@@ -43,11 +43,17 @@ bool gemv_batch_eligible(const sss_qtensor_t& t, const uint16_t* x, int batch, c
 cudaError_t launch_gemv_batch(const sss_qtensor_t& t, const uint16_t* x, int batch, float* y,
                               uint32_t* status, cudaStream_t stream);
 
+// matrices of one sss_gemm_multi call (sharing X)
+constexpr int kMaxGemmJobs = 4;
 size_t gemm_workspace_bytes(const sss_qtensor_t& t, int64_t m);
+size_t gemm_multi_workspace_bytes(const sss_qtensor_t* const* ts, int count, int64_t m);
 size_t gemm_workspace_min_bytes(const sss_qtensor_t& t, int64_t m);
 cudaError_t launch_gemm(const sss_qtensor_t& t, const uint16_t* x, int64_t m,
                         float* y, void* workspace, size_t ws_bytes, uint32_t* status,
                         cudaStream_t stream, bool act_q8 = false);
+cudaError_t launch_gemm_multi(const sss_qtensor_t* const* ts, float* const* ys, int count,
+                              const uint16_t* x, int64_t m, void* workspace, size_t ws_bytes,
+                              uint32_t* status, cudaStream_t stream, bool act_q8);
 
 cudaError_t launch_act_q8(const uint16_t* x, int64_t rows, int64_t k, int8_t* q, uint16_t* d,
                           uint32_t* status, cudaStream_t stream);

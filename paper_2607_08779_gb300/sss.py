@@ -33,6 +33,7 @@ STATUS_NAMES = {0: "SSS_OK", 1: "SSS_E_ARG", 2: "SSS_E_UNSUPPORTED", 3: "SSS_E_A
 EXPORTS = ("sss_codes_bytes", "sss_status_string", "sss_last_error", "sss_quantize",
            "sss_dequantize", "sss_gemv", "sss_gemv_multi", "sss_gemm", "sss_workspace_bytes",
            "sss_gemm_noalloc", "sss_gemm_noalloc_max_scratch_bytes", "sss_test_set_stall",
+           "sss_gemm_multi", "sss_gemm_multi_workspace_bytes",
            "sss_gemm_q8", "sss_quantize_act_q8", "sss_sign_diagnostics", "sss_hadamard",
            "sss_quantize_rotated", "sss_quantize_lsq")
 
@@ -107,6 +108,11 @@ def load(build_if_needed: bool = True):
         L.sss_gemv_multi.restype = i32
         L.sss_gemm.argtypes = [P, vp, i64, vp, vp, sz, vp, vp]
         L.sss_gemm.restype = i32
+        L.sss_gemm_multi.argtypes = [ctypes.POINTER(P), ctypes.POINTER(vp), i32, vp, i64, vp, sz,
+                                     vp, vp]
+        L.sss_gemm_multi.restype = i32
+        L.sss_gemm_multi_workspace_bytes.argtypes = [ctypes.POINTER(P), i32, i64]
+        L.sss_gemm_multi_workspace_bytes.restype = sz
         L.sss_workspace_bytes.argtypes = [P, i64, i32]
         L.sss_workspace_bytes.restype = sz
         L.sss_gemm_noalloc.argtypes = [P, vp, i64, vp, vp, vp]
@@ -356,6 +362,46 @@ def _gemm(fn: str, qt: QTensor, x, y, workspace, dev_status, stream):
 def sss_gemm(qt: QTensor, x, y=None, workspace=None, dev_status=None, stream=None):
     """Y [m, n] fp32 = X [m, k] (bf16) @ dequant(qt)^T on the tensor cores."""
     return _gemm("sss_gemm", qt, x, y, workspace, dev_status, stream)
+
+
+def sss_gemm_multi_workspace_bytes(qts, m: int) -> int:
+    """Workspace bytes for sss_gemm_multi over these tensors at m tokens."""
+    descs = [qt.desc() for qt in qts]
+    parr = (ctypes.POINTER(QTensorDesc) * len(qts))(*[ctypes.pointer(d) for d in descs])
+    return int(load().sss_gemm_multi_workspace_bytes(parr, len(qts), m))
+
+
+def sss_gemm_multi(qts, x, ys=None, workspace=None, dev_status=None, stream=None):
+    """Y_j [m, n_j] fp32 = X [m, k] (bf16) @ dequant(qt_j)^T for 1..4 matrices
+    sharing X, in one launch."""
+    import torch
+
+    fn = "sss_gemm_multi"
+    m = x.shape[0]
+    if ys is None:
+        ys = [torch.empty((m, qt.n), dtype=torch.float32, device=x.device) for qt in qts]
+    if len(ys) != len(qts):
+        raise SssError(fn, 1, "one output per matrix")
+    for qt, y in zip(qts, ys):
+        _need(fn, "x", x, torch.bfloat16, m * qt.k)
+        _need(fn, "y", y, torch.float32, m * qt.n)
+        _need_qtensor(fn, qt)
+        _on_device(fn, y=y, codes=qt.codes, scales=qt.scales, mins=qt.mins)
+    _need(fn, "workspace", workspace, torch.uint8, optional=True)
+    _need_status(fn, dev_status)
+    _on_device(fn, x=x, workspace=workspace, dev_status=dev_status)
+    if workspace is None:
+        need = sss_gemm_multi_workspace_bytes(qts, m)
+        if need > 0:
+            workspace = torch.empty(need, dtype=torch.uint8, device=x.device)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    descs = [qt.desc() for qt in qts]
+    parr = (ctypes.POINTER(QTensorDesc) * len(qts))(*[ctypes.pointer(d) for d in descs])
+    yarr = (ctypes.c_void_p * len(qts))(*[_ptr(y) for y in ys])
+    st = load().sss_gemm_multi(parr, yarr, len(qts), _ptr(x), m, _ptr(workspace), ws_bytes,
+                               _ptr(dev_status), _stream(stream))
+    _check(fn, st)
+    return ys
 
 
 def sss_gemm_q8(qt: QTensor, x, y=None, workspace=None, dev_status=None, stream=None):

@@ -81,6 +81,38 @@ def test_gemv_gemm_argument_checks():
     assert L.sss_quantize(ctypes.c_void_p(4096), ctypes.byref(_desc(n=0)), None, None, None) == 0
 
 
+def test_gemm_multi_argument_checks():
+    L = sss.load()
+    P = ctypes.POINTER(sss.QTensorDesc)
+
+    def call(descs, ys, m=64, x=4096, ws=None, ws_bytes=0, count=None):
+        parr = (P * max(len(descs), 1))(*[ctypes.pointer(d) for d in descs])
+        yarr = (ctypes.c_void_p * max(len(ys), 1))(*ys)
+        n = len(descs) if count is None else count
+        return L.sss_gemm_multi(parr, yarr, n, ctypes.c_void_p(x), m, ws, ws_bytes, None, None)
+
+    a, b = _desc(n=64), _desc(n=32)
+    ys = [8192, 16384]
+    assert call([a, b], ys, count=0) == 1
+    assert call([a, b], ys, count=5) == 1
+    assert call([a, _desc(k=512)], ys) == 1           # k differs
+    assert call([a, _desc(q=2)], ys) == 1             # q differs
+    assert call([a, _desc(grid=0)], ys) == 1          # grid differs
+    assert call([a, _desc(n=30)], ys) == 2            # n % 4 != 0
+    assert call([a, b], [8192, 16388]) == 3           # y not 16-byte aligned
+    assert call([a, b], ys, x=4104) == 3              # x not 16-byte aligned
+    assert call([a, b], ys, m=-1) == 1
+    assert call([a, b], ys) == 5                      # no workspace for the fp16 X
+    # empty calls touch nothing
+    assert call([a, b], ys, m=0) == 0
+    assert call([_desc(n=0), _desc(n=0)], [0, 0]) == 0
+    # sizing: at least the fp16 copy of X; 0 for a bad call
+    parr = (P * 2)(ctypes.pointer(a), ctypes.pointer(b))
+    assert L.sss_gemm_multi_workspace_bytes(parr, 2, 64) >= 64 * 256 * 2
+    assert L.sss_gemm_multi_workspace_bytes(parr, 0, 64) == 0
+    assert L.sss_gemm_multi_workspace_bytes(parr, 2, -1) == 0
+
+
 def test_binding_checks_what_a_pointer_cannot_carry():
     """The Python binding rejects tensors the C ABI would misread (wrong
     dtype, strided, wrong element count, host memory) with SSS_E_ARG before
