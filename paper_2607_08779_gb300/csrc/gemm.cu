@@ -737,8 +737,9 @@ int split_for(int64_t k, int64_t rt, int64_t m, size_t ws, int bn, int64_t tiles
 // dequantised for twice the tokens, and a k-block's MMAs take about as long
 // at N = 256 as at N = 128).  Otherwise, when each split keeps at least 64
 // k-blocks, 256-token tiles with K split over as many CTAs as fill the SMs;
-// else 128-token tiles, split (at least 8 k-blocks each) when they leave
-// SMs idle.  The tile's last split sums all partials alone, so a split pays
+// else 256-token tiles unsplit when 128-token tiles would need a second
+// wave; else 128-token tiles, split (at least 8 k-blocks each) when they
+// leave SMs idle.  The tile's last split sums all partials alone, so a split pays
 // only with enough k-blocks behind it.  (Two half-size CTAs per SM, one
 // dequantising set each, measured slower than one full CTA: their rings are
 // half as deep.)  rt: the row tiles of all the call's matrices.
@@ -749,6 +750,9 @@ GemmPlan plan_gemm(int64_t rt, int64_t k, int64_t m, size_t ws) {
     if (tiles >= sms) return {256, 2, 1};
     const int split = split_for(k, rt, m, ws, 256, tiles, 64);
     if (split >= 2) return {256, 2, split};
+    // 128-token tiles would take a second wave (each CTA the whole k-range
+    // again) where 256-token tiles take one
+    if (rt * ((m + 127) / 128) > sms) return {256, 2, 1};
   }
   const int64_t tiles = rt * ((m + 127) / 128);
   if (tiles >= sms) return {128, 2, 1};

@@ -66,15 +66,16 @@ def test_gemm_multi_groups(g):
 
 def test_gemm_multi_llama_qkv():
     # q/k/v of a Llama3-8B layer at 512 tokens: whole output rows of three
-    # tokens against the oracle; q alone takes the same plan (128-token
-    # tiles, K unsplit), so its output is the same bits
+    # tokens against the oracle, and every token of q against q alone (which
+    # takes 128-token tiles where the fused call takes 256-token ones)
     dims = inputs.LLAMA3_8B_LAYER
     ns = [dims[nm][0] for nm in ("q_proj", "k_proj", "v_proj")]
     k = dims["q_proj"][1]
     qts, X, Ys = run_multi(ns, k, 512, 4, 32, sss.GRID_SIGNED_SYM, 500, tokens=[0, 301, 511])
     Yq = sss.sss_gemm(qts[0], X)
     torch.cuda.synchronize()
-    assert torch.equal(Yq, Ys[0])
+    err = rel_err_per_row(Ys[0].cpu().numpy(), Yq.cpu().numpy().astype(np.float64))
+    assert err.max() <= REL_TOL
 
 
 def test_gemm_multi_llama_gate_up_matches_single_calls():
