@@ -12,7 +12,9 @@
 // 65504).  tcgen05.mma kind::f16 takes both operands in fp16 and accumulates
 // in fp32 in tensor memory.
 //
-// Structure (one CTA per 128-row x BN-token output tile, 18 warps):
+// Structure (one CTA per 128-row x BN-token output tile, 18 warps; the
+// row tiles may belong to up to four matrices that share X, one launch for
+// a fused q/k/v or gate/up projection):
 //   warp 0     TMA producer for the fp16 activation tile (128B swizzle) and
 //              owner of the tensor-memory allocation;
 //   warp 1     a single elected thread issues tcgen05.mma (M=128, N=BN,
