@@ -6,8 +6,8 @@ import torch
 import oracle
 from paper_2607_08779_gb300 import inputs, sss
 
-# the benchmark spec tolerance for GEMV/GEMM outputs vs the fp64 oracle: max relative
-# error 1e-3, read per output vector as max|y - y_ref| / max|y_ref|.
+# Output tolerance of the GEMV and GEMM against the fp64 oracle: relative
+# error 1e-3 per output vector, max|y - y_ref| / max|y_ref|.
 REL_TOL = 1e-3
 
 DEV = "cuda"
