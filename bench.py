@@ -586,6 +586,30 @@ def _oracle_quantize_worker(job):
     return oracle_quantize_rate(*job)
 
 
+def oracle_gemm_rate(codes, scales, n_rows, k, q, xbits, seconds):
+    """FLOP/s the oracle GEMM (dequantise a block of packed rows, then the
+    fp64 matmul with the tokens xbits) sustains on this host (one process),
+    over row blocks of the sample for `seconds`."""
+    import oracle
+
+    rows_per_call = 64
+    m = xbits.shape[0]
+    flops, t0, r0 = 0, time.perf_counter(), 0
+    while time.perf_counter() - t0 < seconds:
+        r1 = min(n_rows, r0 + rows_per_call)
+        What = oracle.dequantize(codes, scales, None, n_rows, k, q, GROUP, oracle.GRID_SIGNED_SYM,
+                                 rows=(r0, r1 - r0))
+        oracle.matmul_f64(What, xbits)
+        flops += 2 * (r1 - r0) * k * m
+        r0 = 0 if r1 >= n_rows else r1
+    el = time.perf_counter() - t0
+    return flops / el, flops, el
+
+
+def _oracle_gemm_worker(job):
+    return oracle_gemm_rate(*job)
+
+
 def host_cores() -> int:
     try:
         return max(1, len(os.sched_getaffinity(0)))
@@ -595,7 +619,9 @@ def host_cores() -> int:
 
 def cpu_baseline(wl, seconds: float, cores: int):
     """The oracle's GEMV, as it stands, on the host cores, on a bounded
-    sample of the same workload (rows of the layer-0 gate_proj at q=4)."""
+    sample of the same workload (rows of the layer-0 gate_proj at q=4); and
+    beside it the oracle quantizer and the oracle GEMM on samples of their
+    phases."""
     mi = [name for name, _ in wl.shapes].index("gate_proj")
     qt = wl.stack[4][0][mi]
     n, k = qt.n, qt.k
@@ -604,6 +630,9 @@ def cpu_baseline(wl, seconds: float, cores: int):
     xbits = wl.x[k].cpu().view(wl.torch.int16).numpy().view(np.uint16)
     # the quantize phase's oracle: rows of the fresh fp32 gate_proj at q=4
     wq = wl.fresh[0][mi][:256].cpu().numpy()
+    # the GEMM phase's oracle: the same packed rows against 16 of its tokens
+    gtok = 16
+    Xs = wl.X[k][:gtok].cpu().view(wl.torch.int16).numpy().view(np.uint16)
     pool = oracle_pool(cores)
     if pool is None:
         cores = 1
@@ -611,16 +640,21 @@ def cpu_baseline(wl, seconds: float, cores: int):
         gbs, gbs1, rows, el = oracle_gemv_rate_cores(pool, cores, codes, scales, codes.shape[0],
                                                      k, 4, xbits, seconds)
         qsec = max(1.0, seconds / 2)
+        gjob = (codes, scales, codes.shape[0], k, 4, Xs, qsec)
         if pool is None:
             qres = [oracle_quantize_rate(wq, 4, qsec)]
+            gres = [oracle_gemm_rate(*gjob)]
         else:
             qres = pool.map(_oracle_quantize_worker, [(wq, 4, qsec)] * cores)
+            gres = pool.map(_oracle_gemm_worker, [gjob] * cores)
     finally:
         if pool is not None:
             pool.close()
             pool.join()
     qwall = max(e for _, _, e in qres)
     qdone = sum(d for _, d, _ in qres)
+    gwall = max(e for _, _, e in gres)
+    gdone = sum(d for _, d, _ in gres)
     return {"value": round(gbs, 4), "unit": "GB/s", "cores": cores, "kind": "oracle",
             "single_core_value": round(gbs1, 4),
             "sample": f"{rows} rows of gate_proj (14336x4096) at q=4 g=32, batch 1: "
@@ -629,7 +663,13 @@ def cpu_baseline(wl, seconds: float, cores: int):
                          "cores": cores, "single_core_value": round(qres[0][0] / 1e9, 6),
                          "sample": f"{qdone} weights: 256 rows of the fresh fp32 gate_proj "
                                    f"(256x4096) at q=4 g=32, signed grid, {cores} processes x "
-                                   f"{qwall:.1f} s of the single-threaded oracle quantizer"}}
+                                   f"{qwall:.1f} s of the single-threaded oracle quantizer"},
+            "gemm": {"value": round(gdone / gwall / 1e12, 9), "unit": "TFLOP/s", "cores": cores,
+                     "single_core_value": round(gres[0][0] / 1e12, 9),
+                     "sample": f"{gdone} FLOPs: blocks of 64 packed gate_proj rows at q=4 g=32 "
+                               f"dequantised, then the fp64 matmul with {gtok} tokens of the "
+                               f"prefill X; {cores} processes x {gwall:.1f} s of the "
+                               f"single-threaded oracle GEMM"}}
 
 
 def run_reference(args):
