@@ -113,6 +113,31 @@ def test_gemm_multi_argument_checks():
     assert L.sss_gemm_multi_workspace_bytes(parr, 2, -1) == 0
 
 
+def test_gemm_workspace_follows_the_tile_plan():
+    # The workspace holds the fp16 X, plus the split-K partial tiles when the
+    # preferred plan splits K (the plan depends only on shapes and the SM
+    # count; without a GPU the library assumes 148 SMs, which gives the same
+    # plans here as the GB300's 152).
+    L = sss.load()
+    P = ctypes.POINTER(sss.QTensorDesc)
+    m, k = 512, 4096
+    x16 = m * k * 2
+
+    def ws(*ns):
+        ds = [_desc(n=n, k=k) for n in ns]
+        parr = (P * len(ds))(*[ctypes.pointer(d) for d in ds])
+        return L.sss_gemm_multi_workspace_bytes(parr, len(ds), m)
+
+    # fused q/k/v: 48 row tiles; 256-token tiles make 96 CTAs in one wave,
+    # 128-token ones would need two, so it runs unsplit
+    assert ws(4096, 1024, 1024) == x16
+    # k_proj alone: 32 CTAs of 128-token tiles, K split over the idle SMs
+    assert ws(1024) > x16
+    # the one-matrix helper agrees with the multi one
+    d = _desc(n=1024, k=k)
+    assert L.sss_workspace_bytes(ctypes.byref(d), m, sss.OP_GEMM) == ws(1024)
+
+
 def test_binding_checks_what_a_pointer_cannot_carry():
     """The Python binding rejects tensors the C ABI would misread (wrong
     dtype, strided, wrong element count, host memory) with SSS_E_ARG before
